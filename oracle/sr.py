@@ -163,6 +163,12 @@ class SpeculativeRejection:
                 self.status[i] = REJECTED
                 self._release(i)
         self.rounds.append(Round(g, batch, rewards, k, k != k0, rc, np.asarray(mask, dtype=bool)))
+        self.snapshots.append(self._snapshot(g))
+
+    def _snapshot(self, g):
+        """Copy of the bookkeeping state (for comparisons; no effect on the run)."""
+        return dict(step=g, status=list(self.status), lengths=[len(t) for t in self.tokens],
+                    page_tables=[list(p) for p in self.page_table], free_stack=list(self.pool.stack))
 
     # -- Algorithm 1 ----------------------------------------------------------------
     def run(self) -> Result:
@@ -171,6 +177,7 @@ class SpeculativeRejection:
         self.tokens: List[List[int]] = [[] for _ in range(N)]
         self.final_reward = np.full(N, np.nan, np.float32)
         self.rounds: List[Round] = []
+        self.snapshots: List[dict] = []
         self.gen_tokens = 0
         self.rm_tokens = P
         shared = [self.pool.pop() for _ in range(P // PAGE)]

@@ -1,0 +1,504 @@
+// Attention for the generator's decode steps and for reward-model / prompt prefill.
+//
+// softmax(q k^T / sqrt(dh)) v per query head, GQA (query head j reads kv head j / (Hq / Hkv)),
+// causal, optional sliding window -- the attention of the decoder-only models of Section 3.
+//
+// Decode (k_decode_attn): one CTA per (kv head, slot, KV split of 512 positions); the CTA serves
+// the G query heads of its kv head, so each K/V byte is read once per group.  A token's K (and V)
+// row of dh elements is read by dh*size/16 threads with one 16-byte load each (fully coalesced
+// within the 4 KB (bf16, dh 128) page block of that head); token groups stride over the split;
+// scores are reduced with warp shuffles and folded into per-group online-softmax state, merged
+// through shared memory at the end.  Splits are a fixed number of positions, so a candidate's
+// result does not depend on the batch it is in; a combine kernel merges split partials.
+//
+// Prefill (k_prefill_attn): flash-attention style over packed variable-length sequences with a
+// shared prefix (the prompt's KV) -- 64 query rows x one head per CTA, 64-key blocks staged by
+// cp.async, bf16 mma.sync m16n8k16 with fp32 accumulation, online softmax in registers.
+#include "common.cuh"
+
+namespace sr {
+namespace {
+
+constexpr int SPLIT = 512;  // KV positions per decode split
+
+template <typename T, int DH, int G>
+__global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, const T* __restrict__ pool,
+                                                     const int* __restrict__ pt, int pt_stride,
+                                                     const int* __restrict__ slot_ids, const int* __restrict__ lens,
+                                                     int Hkv, float scale_log2, int window, int max_splits,
+                                                     T* __restrict__ out, float* __restrict__ part) {
+  constexpr int VE = 16 / sizeof(T);  // elements per 16-byte vector
+  constexpr int TPT = DH / VE;        // threads per token
+  constexpr int NG = 128 / TPT;       // token groups per CTA
+  static_assert(TPT >= 1 && TPT <= 32 && 32 % TPT == 0, "head_dim / dtype combination");
+  __shared__ float s_m[NG][G], s_l[NG][G];
+  __shared__ float s_acc[NG][G][DH];
+
+  const int h = blockIdx.x, s = blockIdx.y, split = blockIdx.z;
+  const int Hq = Hkv * G;
+  const int L = lens[s];
+  const int t_lo = window > 0 ? max(0, L - window) : 0;
+  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  if (split >= nsplit) return;
+  const int t_begin = t_lo + split * SPLIT, t_end = min(L, t_begin + SPLIT);
+  const int tid = threadIdx.x, grp = tid / TPT, sub = tid % TPT, d0 = sub * VE;
+  const int id = slot_ids[s];
+
+  float qv[G][VE];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const T* qp = q + ((size_t)s * Hq + h * G + g) * DH + d0;
+    const uint4 raw = *reinterpret_cast<const uint4*>(qp);
+    const T* e = reinterpret_cast<const T*>(&raw);
+#pragma unroll
+    for (int i = 0; i < VE; ++i) qv[g][i] = to_f(e[i]) * scale_log2;
+  }
+  float m[G], l[G], acc[G][VE];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    m[g] = -INFINITY;
+    l[g] = 0.f;
+#pragma unroll
+    for (int i = 0; i < VE; ++i) acc[g][i] = 0.f;
+  }
+  const int* ptrow = pt + (size_t)id * pt_stride;
+  const size_t page_elems = (size_t)2 * Hkv * PAGE * DH;
+  const size_t v_off = (size_t)Hkv * PAGE * DH;
+
+  // The trip count is the same for every thread of the CTA (base is block-uniform), so the
+  // full-warp shuffles below always see all 32 lanes; a group past the end masks its update.
+  for (int base = t_begin; base < t_end; base += NG) {
+    const int t = base + grp;
+    const bool valid = t < t_end;
+    float kf[VE], vf[VE];
+    if (valid) {
+      const int page = ptrow[t / PAGE];
+      const T* kp = pool + (size_t)page * page_elems + ((size_t)h * PAGE + (t % PAGE)) * DH + d0;
+      const uint4 kr = *reinterpret_cast<const uint4*>(kp);
+      const uint4 vr = *reinterpret_cast<const uint4*>(kp + v_off);
+      const T* ke = reinterpret_cast<const T*>(&kr);
+      const T* ve = reinterpret_cast<const T*>(&vr);
+#pragma unroll
+      for (int i = 0; i < VE; ++i) kf[i] = to_f(ke[i]), vf[i] = to_f(ve[i]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < VE; ++i) kf[i] = 0.f, vf[i] = 0.f;
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      float sc = 0.f;
+#pragma unroll
+      for (int i = 0; i < VE; ++i) sc = fmaf(qv[g][i], kf[i], sc);
+#pragma unroll
+      for (int o = TPT / 2; o > 0; o >>= 1) sc += __shfl_xor_sync(0xffffffffu, sc, o);
+      if (!valid) continue;
+      const float mn = fmaxf(m[g], sc);
+      const float corr = exp2f(m[g] - mn);
+      const float p = exp2f(sc - mn);
+      l[g] = l[g] * corr + p;
+#pragma unroll
+      for (int i = 0; i < VE; ++i) acc[g][i] = fmaf(acc[g][i], corr, p * vf[i]);
+      m[g] = mn;
+    }
+  }
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    if (sub == 0) s_m[grp][g] = m[g], s_l[grp][g] = l[g];
+#pragma unroll
+    for (int i = 0; i < VE; ++i) s_acc[grp][g][d0 + i] = acc[g][i];
+  }
+  __syncthreads();
+  for (int idx = tid; idx < G * DH; idx += 128) {
+    const int g = idx / DH, d = idx % DH;
+    float M = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < NG; ++j) M = fmaxf(M, s_m[j][g]);
+    float Lsum = 0.f, O = 0.f;
+#pragma unroll
+    for (int j = 0; j < NG; ++j) {
+      const float w = (s_m[j][g] == -INFINITY) ? 0.f : exp2f(s_m[j][g] - M);
+      Lsum += s_l[j][g] * w;
+      O += s_acc[j][g][d] * w;
+    }
+    const int hq = h * G + g;
+    if (nsplit == 1) {
+      out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
+    } else {
+      float* pp = part + (((size_t)s * Hq + hq) * max_splits + split) * (DH + 2);
+      pp[d] = O;
+      if (d == 0) pp[DH] = M, pp[DH + 1] = Lsum;
+    }
+  }
+}
+
+template <typename T, int DH>
+__global__ void k_decode_combine(const float* __restrict__ part, const int* __restrict__ lens, int Hq, int window,
+                                 int max_splits, T* __restrict__ out) {
+  const int hq = blockIdx.x, s = blockIdx.y, d = threadIdx.x;
+  const int L = lens[s];
+  const int t_lo = window > 0 ? max(0, L - window) : 0;
+  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  if (nsplit <= 1) return;  // written directly by k_decode_attn
+  const float* pp = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
+  float M = -INFINITY;
+  for (int j = 0; j < nsplit; ++j) M = fmaxf(M, pp[j * (DH + 2) + DH]);
+  float Lsum = 0.f, O = 0.f;
+  for (int j = 0; j < nsplit; ++j) {
+    const float w = exp2f(pp[j * (DH + 2) + DH] - M);
+    Lsum += pp[j * (DH + 2) + DH + 1] * w;
+    O += pp[j * (DH + 2) + d] * w;
+  }
+  out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
+}
+
+// ------------------------------------------------------------------------------------------------
+// prefill attention
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst)), "l"(src), "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void ldm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float* c, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+constexpr int BQ = 64, BKV = 64;
+
+template <int DH, int DV>
+__global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q, const bf16* __restrict__ k,
+                                                      const bf16* __restrict__ v, const bf16* __restrict__ kpre,
+                                                      const bf16* __restrict__ vpre, int npre,
+                                                      const int* __restrict__ seq_off,
+                                                      const int* __restrict__ tile_seq,
+                                                      const int* __restrict__ tile_q0, int pos0, int Hq, int Hkv,
+                                                      float scale_log2, int window, bf16* __restrict__ out) {
+  constexpr int LD = DH + 8, LDV = DV + 8;
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  bf16* sQ = reinterpret_cast<bf16*>(smem_raw);
+  bf16* sK = sQ + BQ * LD;
+  bf16* sV = sK + BKV * LD;
+
+  const int tile = blockIdx.x, hq = blockIdx.y, dvo = blockIdx.z * DV;
+  const int j = tile_seq[tile], q0 = tile_q0[tile];
+  const int r0 = seq_off[j], nrows = seq_off[j + 1] - r0;
+  const int hk = hq / (Hq / Hkv);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
+  const size_t qstride = (size_t)Hq * DH, kstride = (size_t)Hkv * DH;
+
+  // Q tile
+  for (int c = tid; c < BQ * (DH / 8); c += 128) {
+    const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+    const bool ok = q0 + row < nrows;
+    const bf16* src = ok ? q + (size_t)(r0 + q0 + row) * qstride + (size_t)hq * DH + col : q;
+    cp_async16(sQ + row * LD + col, src, ok);
+  }
+
+  float o[DV / 8][4];
+#pragma unroll
+  for (int i = 0; i < DV / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  const int qi_a = q0 + warp * 16 + g;  // query index within the sequence (rows g and g + 8)
+  const int qpos[2] = {pos0 + qi_a, pos0 + qi_a + 8};
+  const int qpos_min = pos0 + q0;
+  const int qpos_max = pos0 + min(nrows, q0 + BQ) - 1;
+
+  const int nb_pre = (npre + BKV - 1) / BKV;
+  const int own_keys = min(nrows, q0 + BQ);
+  const int nb_own = (own_keys + BKV - 1) / BKV;
+
+  for (int kb = 0; kb < nb_pre + nb_own; ++kb) {
+    const bool is_pre = kb < nb_pre;
+    const int kbase = is_pre ? kb * BKV : (kb - nb_pre) * BKV;   // key index within its segment
+    const int kcount = is_pre ? min(BKV, npre - kbase) : min(BKV, own_keys - kbase);
+    const int kpos0 = is_pre ? kbase : pos0 + kbase;
+    if (window > 0 && kpos0 + kcount - 1 <= qpos_min - window) continue;  // whole block left of every window
+    if (kpos0 > qpos_max) continue;
+    __syncthreads();  // previous block's smem reads are done
+    const bf16* ksrc = is_pre ? kpre : k + (size_t)r0 * kstride;
+    const bf16* vsrc = is_pre ? vpre : v + (size_t)r0 * kstride;
+    for (int c = tid; c < BKV * (DH / 8); c += 128) {
+      const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+      const bool ok = row < kcount;
+      const bf16* src = ok ? ksrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + col : ksrc;
+      cp_async16(sK + row * LD + col, src, ok);
+    }
+    for (int c = tid; c < BKV * (DV / 8); c += 128) {
+      const int row = c / (DV / 8), col = (c % (DV / 8)) * 8;
+      const bool ok = row < kcount;
+      const bf16* src = ok ? vsrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + dvo + col : vsrc;
+      cp_async16(sV + row * LDV + col, src, ok);
+    }
+    cp_async_wait_all();
+    __syncthreads();
+
+    // S = Q K^T for this warp's 16 rows x 64 keys
+    float sc[BKV / 8][4];
+#pragma unroll
+    for (int i = 0; i < BKV / 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < DH / 16; ++kk) {
+      uint32_t a0, a1, a2, a3;
+      ldm_x4(smem_addr(sQ + (warp * 16 + (lane & 15)) * LD + kk * 16 + (lane >> 4) * 8), a0, a1, a2, a3);
+#pragma unroll
+      for (int np = 0; np < BKV / 16; ++np) {
+        uint32_t b0, b1, b2, b3;
+        ldm_x4(smem_addr(sK + (np * 16 + (lane & 7) + ((lane >> 4) << 3)) * LD + kk * 16 + ((lane >> 3) & 1) * 8), b0,
+               b1, b2, b3);
+        mma16816(sc[2 * np], a0, a1, a2, a3, b0, b1);
+        mma16816(sc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+    // mask, scale, online softmax
+    float bmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int nt = 0; nt < BKV / 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int kidx = nt * 8 + 2 * t4 + (e & 1);
+        const int r = e >> 1;
+        const int kpos = kpos0 + kidx;
+        bool ok = kidx < kcount && kpos <= qpos[r];
+        if (window > 0) ok = ok && kpos > qpos[r] - window;
+        const float x = ok ? sc[nt][e] * scale_log2 : -INFINITY;
+        sc[nt][e] = x;
+        bmax[r] = fmaxf(bmax[r], x);
+      }
+    }
+    float corr[2], base[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      bmax[r] = fmaxf(bmax[r], __shfl_xor_sync(0xffffffffu, bmax[r], 1));
+      bmax[r] = fmaxf(bmax[r], __shfl_xor_sync(0xffffffffu, bmax[r], 2));
+      const float mn = fmaxf(mrow[r], bmax[r]);
+      base[r] = (mn == -INFINITY) ? 0.f : mn;
+      corr[r] = exp2f(mrow[r] - base[r]);
+      mrow[r] = mn;
+    }
+    float psum[2] = {0.f, 0.f};
+#pragma unroll
+    for (int nt = 0; nt < BKV / 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float p = exp2f(sc[nt][e] - base[e >> 1]);
+        sc[nt][e] = p;
+        psum[e >> 1] += p;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) lrow[r] = lrow[r] * corr[r] + psum[r];
+#pragma unroll
+    for (int i = 0; i < DV / 8; ++i) {
+      o[i][0] *= corr[0], o[i][1] *= corr[0];
+      o[i][2] *= corr[1], o[i][3] *= corr[1];
+    }
+    // O += P V
+#pragma unroll
+    for (int kk = 0; kk < BKV / 16; ++kk) {
+      const uint32_t a0 = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+      const uint32_t a1 = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+      const uint32_t a2 = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      const uint32_t a3 = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < DV / 16; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LDV + dp * 16 + (lane >> 4) * 8), b0,
+                 b1, b2, b3);
+        mma16816(o[2 * dp], a0, a1, a2, a3, b0, b1);
+        mma16816(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+  }
+  // finish: full row sums across the quad, normalise, store
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+    lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+  }
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int qi = qi_a + 8 * r;
+    if (qi >= nrows) continue;
+    const float inv = lrow[r] > 0.f ? 1.f / lrow[r] : 0.f;
+    bf16* dst = out + (size_t)(r0 + qi) * qstride + (size_t)hq * DH + dvo;
+#pragma unroll
+    for (int nt = 0; nt < DV / 8; ++nt) {
+      const __nv_bfloat162 h = __floats2bfloat162_rn(o[nt][2 * r] * inv, o[nt][2 * r + 1] * inv);
+      *reinterpret_cast<__nv_bfloat162*>(dst + nt * 8 + 2 * t4) = h;
+    }
+  }
+}
+
+// fp32 models: straightforward prefill attention, one block per (query row, head); scores of the
+// row's visible keys live in shared memory.
+__global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __restrict__ k,
+                                   const float* __restrict__ v, const float* __restrict__ kpre,
+                                   const float* __restrict__ vpre, int npre, const int* __restrict__ seq_off,
+                                   int n_seq, int pos0, int Hq, int Hkv, int dh, float scale, int window,
+                                   float* __restrict__ out) {
+  extern __shared__ float sc[];
+  __shared__ float red[32];
+  const int r = blockIdx.x, hq = blockIdx.y, hk = hq / (Hq / Hkv);
+  int j = 0;
+  while (j + 1 < n_seq && seq_off[j + 1] <= r) ++j;
+  const int r0 = seq_off[j], qi = r - r0, qpos = pos0 + qi;
+  const int nk = npre + qi + 1;
+  const float* qr = q + ((size_t)r * Hq + hq) * dh;
+  float mx = -INFINITY;
+  for (int t = threadIdx.x; t < nk; t += blockDim.x) {
+    const bool pre = t < npre;
+    const int kpos = pre ? t : pos0 + (t - npre);
+    const float* kr = pre ? kpre + ((size_t)t * Hkv + hk) * dh : k + ((size_t)(r0 + t - npre) * Hkv + hk) * dh;
+    float s = 0.f;
+    for (int d = 0; d < dh; ++d) s = fmaf(qr[d], kr[d], s);
+    s *= scale;
+    if (window > 0 && kpos <= qpos - window) s = -INFINITY;
+    sc[t] = s;
+    mx = fmaxf(mx, s);
+  }
+  mx = warp_max(mx);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  __syncthreads();
+  mx = -INFINITY;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) mx = fmaxf(mx, red[w]);
+  float sum = 0.f;
+  for (int t = threadIdx.x; t < nk; t += blockDim.x) {
+    const float p = expf(sc[t] - mx);
+    sc[t] = p;
+    sum += p;
+  }
+  sum = block_sum(sum, red);
+  for (int d = threadIdx.x; d < dh; d += blockDim.x) {
+    float o = 0.f;
+    for (int t = 0; t < nk; ++t) {
+      const bool pre = t < npre;
+      const float* vr = pre ? vpre + ((size_t)t * Hkv + hk) * dh : v + ((size_t)(r0 + t - npre) * Hkv + hk) * dh;
+      o = fmaf(sc[t], vr[d], o);
+    }
+    out[((size_t)r * Hq + hq) * dh + d] = o / sum;
+  }
+}
+
+template <typename T, int DH, int G>
+sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
+                        const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
+                        cudaStream_t st) {
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
+  dim3 grid(Hkv, b, max_splits);
+  k_decode_attn<T, DH, G><<<grid, 128, 0, st>>>((const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
+                                                 scale_log2, window, max_splits, (T*)out, part);
+  SR_LAUNCH();
+  if (max_splits > 1) {
+    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, (T*)out);
+    SR_LAUNCH();
+  }
+  return SR_OK;
+}
+
+template <int DH, int DV>
+sr_status prefill_t(const bf16* q, const bf16* k, const bf16* v, const bf16* kpre, const bf16* vpre, int npre,
+                    const int* seq_off, const int* tile_seq, const int* tile_q0, int n_tiles, int pos0, int Hq,
+                    int Hkv, int window, bf16* out, cudaStream_t st) {
+  const size_t smem = (size_t)(BQ * (DH + 8) + BKV * (DH + 8) + BKV * (DV + 8)) * sizeof(bf16);
+  static bool attr_set = false;
+  if (!attr_set) {
+    SR_CUDA(cudaFuncSetAttribute(k_prefill_attn<DH, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    attr_set = true;
+  }
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
+  dim3 grid(n_tiles, Hq, DH / DV);
+  k_prefill_attn<DH, DV><<<grid, 128, smem, st>>>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, pos0, Hq,
+                                                   Hkv, scale_log2, window, out);
+  SR_LAUNCH();
+  return SR_OK;
+}
+
+}  // namespace
+
+int decode_attention_max_splits(int max_len) { return max_len <= 0 ? 1 : (max_len + SPLIT - 1) / SPLIT; }
+size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits) {
+  return (size_t)b * Hq * max_splits * (dh + 2);
+}
+
+sr_status launch_decode_attention(int dtype, const void* q, const void* pool_layer, const int* pt, int pt_stride,
+                                  const int* ids, const int* lens, int b, int Hq, int Hkv, int dh, int window,
+                                  void* out, float* part, int max_splits, cudaStream_t st) {
+  if (b == 0) return SR_OK;
+  const int G = Hq / Hkv;
+  if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "decode attention: n_heads %% n_kv_heads != 0");
+  if (max_splits > 1 && !part) return set_err(SR_ERR_INVALID_ARG, "decode attention: split partial buffer missing");
+#define SR_DEC(T, D, GG)                                                                                      \
+  if (dh == D && G == GG)                                                                                     \
+    return decode_attn_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
+                                   st);
+  if (dtype == SR_DT_BF16) {
+    SR_DEC(bf16, 128, 4) SR_DEC(bf16, 128, 1) SR_DEC(bf16, 128, 2) SR_DEC(bf16, 128, 8)
+    SR_DEC(bf16, 64, 1) SR_DEC(bf16, 64, 4) SR_DEC(bf16, 32, 1)
+  } else {
+    SR_DEC(float, 32, 1) SR_DEC(float, 32, 2) SR_DEC(float, 32, 4) SR_DEC(float, 64, 1) SR_DEC(float, 128, 1)
+    SR_DEC(float, 8, 1) SR_DEC(float, 8, 2) SR_DEC(float, 8, 4)
+  }
+#undef SR_DEC
+  return set_err(SR_ERR_UNSUPPORTED, "decode attention: head_dim %d with group %d (dtype %d) not built", dh, G, dtype);
+}
+
+sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* kpre,
+                                       const float* vpre, int npre, const int* seq_off, int n_seq, int rows, int pos0,
+                                       int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st) {
+  if (rows == 0) return SR_OK;
+  const int max_keys = npre + rows;
+  const size_t smem = (size_t)max_keys * sizeof(float);
+  if (smem > 200 * 1024) return set_err(SR_ERR_UNSUPPORTED, "fp32 prefill attention: %d keys too many", max_keys);
+  static size_t attr = 48 * 1024;
+  if (smem > attr) {
+    SR_CUDA(cudaFuncSetAttribute(k_prefill_attn_f32, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    attr = smem;
+  }
+  k_prefill_attn_f32<<<dim3(rows, Hq), 128, smem, st>>>(q, k, v, kpre, vpre, npre, seq_off, n_seq, pos0, Hq, Hkv, dh,
+                                                        1.f / sqrtf((float)dh), window, out);
+  SR_LAUNCH();
+  return SR_OK;
+}
+
+sr_status launch_prefill_attention(const bf16* q, const bf16* k, const bf16* v, const bf16* kpre, const bf16* vpre,
+                                   int npre, const int* seq_off, int n_seq, const int* tile_seq, const int* tile_q0,
+                                   int n_tiles, int pos0, int Hq, int Hkv, int dh, int window, bf16* out,
+                                   cudaStream_t st) {
+  (void)n_seq;
+  if (n_tiles == 0) return SR_OK;
+  if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "prefill attention: n_heads %% n_kv_heads != 0");
+  switch (dh) {
+    case 32: return prefill_t<32, 32>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
+    case 64: return prefill_t<64, 64>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
+    case 128: return prefill_t<128, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
+    case 256: return prefill_t<256, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
+  }
+  return set_err(SR_ERR_UNSUPPORTED, "prefill attention: head_dim %d not built", dh);
+}
+
+}  // namespace sr

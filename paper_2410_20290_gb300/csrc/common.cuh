@@ -1,0 +1,183 @@
+// Shared device helpers and host-side declarations of libsr.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "sr.h"
+
+namespace sr {
+
+typedef __nv_bfloat16 bf16;
+constexpr int PAGE = 16;            // positions per KV page
+constexpr int MAX_BATCH = 4096;     // largest N handled by the single-CTA control kernels
+
+// ---------------------------------------------------------------------------------------------
+// error reporting (host)
+// ---------------------------------------------------------------------------------------------
+sr_status set_err(sr_status s, const char* fmt, ...);
+
+#define SR_CUDA(call)                                                                                 \
+  do {                                                                                                \
+    cudaError_t e_ = (call);                                                                          \
+    if (e_ != cudaSuccess)                                                                            \
+      return ::sr::set_err(e_ == cudaErrorMemoryAllocation ? SR_ERR_OOM : SR_ERR_CUDA, "%s:%d %s: %s", \
+                           __FILE__, __LINE__, #call, cudaGetErrorString(e_));                        \
+  } while (0)
+#define SR_LAUNCH() SR_CUDA(cudaGetLastError())
+#define SR_TRY(expr)               \
+  do {                             \
+    sr_status s_ = (expr);         \
+    if (s_ != SR_OK) return s_;    \
+  } while (0)
+
+// ---------------------------------------------------------------------------------------------
+// device helpers
+// ---------------------------------------------------------------------------------------------
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+template <typename T>
+__device__ __forceinline__ T f_to(float x);
+template <>
+__device__ __forceinline__ float f_to<float>(float x) { return x; }
+template <>
+__device__ __forceinline__ bf16 f_to<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// block-wide sum for blockDim.x <= 1024; `red` holds >= 32 floats
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[wid] = v;
+  __syncthreads();
+  float t = (threadIdx.x < nw) ? red[threadIdx.x] : 0.f;
+  if (wid == 0) t = warp_sum(t);
+  if (threadIdx.x == 0) red[0] = t;
+  __syncthreads();
+  return red[0];
+}
+
+// block-wide exclusive scan of ints for blockDim.x <= 1024; returns the total; `tmp` >= 33 ints
+__device__ __forceinline__ int block_excl_scan(int v, int* tmp, int* total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  __syncthreads();
+  if (lane == 31) tmp[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    int s = (lane < nw) ? tmp[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    tmp[lane] = s;  // inclusive scan of warp totals
+  }
+  __syncthreads();
+  int base = (wid > 0) ? tmp[wid - 1] : 0;
+  if (total) *total = tmp[nw - 1];
+  return base + x - v;
+}
+
+// order-preserving map float -> uint32 (-0 folded onto +0, NaN ordered as -inf)
+__device__ __forceinline__ uint32_t float_key(float r) {
+  if (r != r) r = -__int_as_float(0x7f800000);
+  if (r == 0.f) r = 0.f;
+  uint32_t u = __float_as_uint(r);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key_float(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
+// ---------------------------------------------------------------------------------------------
+// host launchers implemented in the kernel files
+// ---------------------------------------------------------------------------------------------
+enum Epi { EPI_F32 = 0, EPI_ADD_F32 = 1, EPI_STORE = 2, EPI_SWIGLU = 3, EPI_GEGLU = 4, EPI_GELU = 5 };
+
+// gemm_tc.cu: bf16 tcgen05 GEMM, C = A W^T; needs sm_100+ tensor memory.
+sr_status gemm_bf16(const bf16* A, const bf16* W, void* C, int M, int N, int K, int epi, cudaStream_t st);
+// gemm_f32.cu: fp32 SIMT GEMM (epilogues EPI_F32, EPI_ADD_F32, EPI_STORE).
+sr_status gemm_f32(const float* A, const float* W, float* C, int M, int N, int K, int epi, cudaStream_t st);
+
+// elementwise.cu
+sr_status launch_embed(int dtype, const void* tok_emb, const void* pos_emb, const int* tokens, const int* positions,
+                       int M, int d, float* x, cudaStream_t st);
+sr_status launch_norm(int dtype, int norm, const float* x, const void* w, const void* b, float eps, int M, int d,
+                      void* out, cudaStream_t st);
+sr_status launch_rope_table(float2* tab, int max_pos, int head_dim, double theta, cudaStream_t st);
+struct KvSink {        // where a layer's new K/V rows go besides the contiguous k/v outputs
+  void* pool_layer;    // this layer's page 0 in the pool, or nullptr
+  const int* page_table;
+  int pt_stride;
+  const int* row_seq;  // page-table row per input row (nullptr: row 0 for every input row)
+};
+sr_status launch_rope_store(int dtype, const float* qkv, int M, const int* positions, const float2* rope, int Hq,
+                            int Hkv, int dh, void* q_out, void* k_out, void* v_out, KvSink sink, cudaStream_t st);
+sr_status launch_act(int dtype, int act, const float* in, int M, int F, void* out, cudaStream_t st);
+sr_status launch_score_head(int dtype, int norm, const float* x, const int* rows, int n, const void* w,
+                            const void* b, float eps, const void* head, int d, float* rewards, cudaStream_t st);
+sr_status launch_copy_page(int dtype, void* pool, long long layer_stride_elems, int n_layers, int page_elems,
+                           int src_page, const int* dst_pages, int n_dst, cudaStream_t st);
+
+// sample.cu
+sr_status launch_sample(const float* logits, long long ld, int b, int V, const int* orig_ids, const int* steps,
+                        uint64_t seed, float temperature, float eos_bias, int eos_id, int* tokens_out,
+                        int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st);
+
+// attention.cu
+sr_status launch_decode_attention(int dtype, const void* q, const void* pool_layer, const int* page_table,
+                                  int pt_stride, const int* slot_ids, const int* lens, int b, int Hq, int Hkv, int dh,
+                                  int window, void* out, float* part, int max_splits, cudaStream_t st);
+int decode_attention_max_splits(int max_len);
+size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits);
+sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* k_pre,
+                                       const float* v_pre, int n_pre, const int* seq_off, int n_seq, int rows,
+                                       int pos0, int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st);
+sr_status launch_prefill_attention(const bf16* q, const bf16* k, const bf16* v, const bf16* k_pre,
+                                   const bf16* v_pre, int n_pre, const int* seq_off, int n_seq, const int* tile_seq,
+                                   const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
+                                   bf16* out, cudaStream_t st);
+
+// select.cu -- device control words and candidate states
+enum Ctrl { C_NLIVE = 0, C_TOP, C_NRSET, C_ERR, C_PEAK, C_K, C_KRAISED, C_NACC, C_BEST, C_NPOOL, C_N };
+enum Status { ST_LIVE = 0, ST_PENDING = 1, ST_DONE = 2, ST_REJECTED = 3, ST_WAITING = 4 };
+enum CtlErr { E_POOL_EMPTY = 1, E_STATE = 2 };
+sr_status ctl_pool_init(int* free_stack, int n_pages, int* ctrl, cudaStream_t st);
+sr_status ctl_prompt_pages(int* free_stack, int* ctrl, int n_sh, int has_tail, int template_page, int* prompt_row,
+                           cudaStream_t st);
+sr_status ctl_admit(int start, int count, int n_sh, int has_tail, const int* prompt_row, int* pt, int max_pages,
+                    int* len, int* status, int* live, int* rset, const int* free_stack, int* ctrl, int* tail_dst,
+                    cudaStream_t st);
+sr_status ctl_step_begin(int P, const int* live, int* ctrl, const int* len, int* pt, int max_pages,
+                         const int* free_stack, const int* tok, int max_new, int* tok_in, int* pos_in, int* kv_len,
+                         cudaStream_t st);
+sr_status ctl_step_end(int P, int n_sh, int* live, int* ctrl, const int* len, const int* status, const int* pt,
+                       int max_pages, int* free_stack, cudaStream_t st);
+sr_status ctl_round(int P, int n_sh, float alpha, int pool_need, const float* rewards, int* rset, int* live,
+                    int* ctrl, float* ctrlf, int* status, const int* len, float* reward_final, const int* pt,
+                    int max_pages, int* free_stack, uint8_t* mask_out, cudaStream_t st);
+sr_status ctl_mark_done(const int* ids, const float* r, int n, int* status, float* reward_final, cudaStream_t st);
+sr_status ctl_final(int N, const int* status, const float* reward_final, const int* tok, int max_new, const int* len,
+                    int* out_tokens, int* out_len, float* out_score, int* ctrl, cudaStream_t st);
+sr_status launch_rcut(const float* rewards, int b, float alpha, int k_override, float* r_cut_out, uint8_t* mask_out,
+                      cudaStream_t st);
+
+}  // namespace sr

@@ -1,0 +1,1084 @@
+// libsr runtime: model loading, workspace, the generator / reward-model forward passes, and the
+// Speculative Rejection controller (Algorithm 1, Section 4.2) behind the C ABI of sr.h.
+//
+// Host code here only enqueues kernels and reads a handful of control words per step (live
+// count, free pages) to size the next launch; every step of the method runs on the device:
+// embedding, norms, GEMMs, RoPE + paged KV append, attention, sampling, partial-reward scoring,
+// the r_cut radix select, compaction and page release.
+#include <algorithm>
+#include <chrono>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+
+namespace sr {
+
+static thread_local std::string g_msg;
+
+sr_status set_err(sr_status s, const char* fmt, ...) {
+  char buf[1024];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_msg = buf;
+  return s;
+}
+
+int* gemm_error_word();
+
+namespace {
+
+template <typename T>
+sr_status grow(T*& p, size_t& cap, size_t n) {
+  if (n <= cap && p) return SR_OK;
+  if (p) cudaFree(p);
+  p = nullptr;
+  cap = 0;
+  SR_CUDA(cudaMalloc(reinterpret_cast<void**>(&p), std::max<size_t>(n, 1) * sizeof(T)));
+  cap = n;
+  return SR_OK;
+}
+
+template <typename T>
+sr_status grow_host(T*& p, size_t& cap, size_t n) {
+  if (n <= cap && p) return SR_OK;
+  if (p) cudaFreeHost(p);
+  p = nullptr;
+  cap = 0;
+  SR_CUDA(cudaMallocHost(reinterpret_cast<void**>(&p), std::max<size_t>(n, 1) * sizeof(T)));
+  cap = n;
+  return SR_OK;
+}
+
+double now_ms() {
+  return std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now().time_since_epoch()).count();
+}
+
+// -------------------------------------------------------------------------------------------------
+// model
+// -------------------------------------------------------------------------------------------------
+struct LayerW {
+  void *attn_w, *attn_b, *wqkv, *wo, *mlp_w, *mlp_b, *wgu, *wdown;
+};
+
+struct Model {
+  sr_model_desc d{};
+  int esz = 2;
+  char* blob = nullptr;
+  void *tok_emb = nullptr, *pos_emb = nullptr, *final_w = nullptr, *final_b = nullptr, *lm_head = nullptr,
+       *score_head = nullptr;
+  std::vector<LayerW> L;
+  float2* rope = nullptr;
+  bool gated() const { return d.act != SR_ACT_GELU; }
+  int qkv_dim() const { return (d.n_heads + 2 * d.n_kv_heads) * d.head_dim; }
+  size_t kv_tok_elems() const { return (size_t)d.n_kv_heads * d.head_dim; }
+};
+
+sr_status check_desc(const sr_model_desc* m, const char* who) {
+  if (!m) return set_err(SR_ERR_INVALID_ARG, "%s: null descriptor", who);
+  if (m->n_layers < 1 || m->d_model < 1 || m->n_heads < 1 || m->n_kv_heads < 1 || m->head_dim < 2 ||
+      m->ffn_dim < 1 || m->vocab < 1 || m->max_pos < 1 || m->window < 0)
+    return set_err(SR_ERR_INVALID_ARG, "%s: non-positive dimension", who);
+  if (m->norm != SR_NORM_RMS && m->norm != SR_NORM_LAYER) return set_err(SR_ERR_INVALID_ARG, "%s: norm", who);
+  if (m->act < SR_ACT_SWIGLU || m->act > SR_ACT_GEGLU) return set_err(SR_ERR_INVALID_ARG, "%s: act", who);
+  if (m->pos != SR_POS_ROPE && m->pos != SR_POS_LEARNED) return set_err(SR_ERR_INVALID_ARG, "%s: pos", who);
+  if (m->dtype != SR_DT_F32 && m->dtype != SR_DT_BF16) return set_err(SR_ERR_INVALID_ARG, "%s: dtype", who);
+  if (m->n_heads % m->n_kv_heads) return set_err(SR_ERR_UNSUPPORTED, "%s: n_heads %% n_kv_heads != 0", who);
+  if (m->head_dim % 2) return set_err(SR_ERR_UNSUPPORTED, "%s: odd head_dim", who);
+  if (m->ffn_dim % 32) return set_err(SR_ERR_UNSUPPORTED, "%s: ffn_dim %% 32 != 0", who);
+  if (m->dtype == SR_DT_BF16) {
+    if (m->d_model % 64 || m->ffn_dim % 64 || m->vocab % 32 || (m->n_heads * m->head_dim) % 64)
+      return set_err(SR_ERR_UNSUPPORTED, "%s: bf16 needs d_model, ffn_dim, n_heads*head_dim %% 64 == 0 and vocab %% 32 == 0",
+                     who);
+    if (m->head_dim != 32 && m->head_dim != 64 && m->head_dim != 128 && m->head_dim != 256)
+      return set_err(SR_ERR_UNSUPPORTED, "%s: head_dim %d (bf16 needs 32/64/128/256)", who, m->head_dim);
+  }
+  return SR_OK;
+}
+
+// Copy one model's blob (host or device; densely packed in the sr.h order) into an aligned
+// device allocation; gate/up rows are interleaved in blocks of 32 for the fused GLU epilogue.
+sr_status load_model(Model& M, const sr_model_desc* d, const void* src) {
+  M.d = *d;
+  M.esz = d->dtype == SR_DT_BF16 ? 2 : 4;
+  const size_t D = d->d_model, F = d->ffn_dim, V = d->vocab, E = M.esz;
+  const bool ln = d->norm == SR_NORM_LAYER;
+  struct T {
+    size_t elems;
+    void** dst;
+    int kind;  // 0 plain, 1 gate (interleave into wgu), 2 up
+  };
+  std::vector<T> ts;
+  M.L.assign(d->n_layers, LayerW{});
+  ts.push_back({V * D, &M.tok_emb, 0});
+  if (d->pos == SR_POS_LEARNED) ts.push_back({(size_t)d->max_pos * D, &M.pos_emb, 0});
+  for (auto& l : M.L) {
+    ts.push_back({D, &l.attn_w, 0});
+    if (ln) ts.push_back({D, &l.attn_b, 0});
+    ts.push_back({(size_t)((d->n_heads + 2 * d->n_kv_heads) * d->head_dim) * D, &l.wqkv, 0});
+    ts.push_back({D * (size_t)(d->n_heads * d->head_dim), &l.wo, 0});
+    ts.push_back({D, &l.mlp_w, 0});
+    if (ln) ts.push_back({D, &l.mlp_b, 0});
+    if (d->act != SR_ACT_GELU) {
+      ts.push_back({F * D, &l.wgu, 1});
+      ts.push_back({F * D, &l.wgu, 2});
+    } else {
+      ts.push_back({F * D, &l.wgu, 0});
+    }
+    ts.push_back({D * F, &l.wdown, 0});
+  }
+  ts.push_back({D, &M.final_w, 0});
+  if (ln) ts.push_back({D, &M.final_b, 0});
+  if (d->has_lm_head) ts.push_back({V * D, &M.lm_head, 0});
+  if (d->has_scalar_head) ts.push_back({D, &M.score_head, 0});
+
+  // destination layout: every tensor 256-byte aligned; a gated layer's gate+up share one [2F][D] slot
+  size_t total = 0;
+  std::vector<size_t> dst_off(ts.size());
+  for (size_t i = 0; i < ts.size(); ++i) {
+    if (ts[i].kind == 2) {
+      dst_off[i] = dst_off[i - 1];
+      continue;
+    }
+    total = (total + 255) & ~size_t(255);
+    dst_off[i] = total;
+    total += ts[i].elems * (ts[i].kind == 1 ? 2 : 1) * E;
+  }
+  SR_CUDA(cudaMalloc(&M.blob, total));
+  size_t soff = 0;
+  const char* s = static_cast<const char*>(src);
+  for (size_t i = 0; i < ts.size(); ++i) {
+    char* dst = M.blob + dst_off[i];
+    *ts[i].dst = dst;
+    const size_t bytes = ts[i].elems * E;
+    if (ts[i].kind == 0) {
+      SR_CUDA(cudaMemcpy(dst, s + soff, bytes, cudaMemcpyDefault));
+    } else {
+      // rows of block j (32 rows of D) land at rows 64j (gate) or 64j + 32 (up)
+      const size_t row_bytes = D * E;
+      char* base = dst + (ts[i].kind == 2 ? 32 * row_bytes : 0);
+      SR_CUDA(cudaMemcpy2D(base, 64 * row_bytes, s + soff, 32 * row_bytes, 32 * row_bytes, F / 32,
+                           cudaMemcpyDefault));
+    }
+    soff += bytes;
+  }
+  if (d->pos == SR_POS_ROPE) {
+    SR_CUDA(cudaMalloc(&M.rope, (size_t)d->max_pos * (d->head_dim / 2) * sizeof(float2)));
+    SR_TRY(launch_rope_table(M.rope, d->max_pos, d->head_dim, (double)d->rope_theta, 0));
+  }
+  SR_CUDA(cudaDeviceSynchronize());
+  return SR_OK;
+}
+
+void free_model(Model& M) {
+  if (M.blob) cudaFree(M.blob);
+  if (M.rope) cudaFree(M.rope);
+  M.blob = nullptr;
+  M.rope = nullptr;
+}
+
+// -------------------------------------------------------------------------------------------------
+// per-model workspace (rows = tokens processed together)
+// -------------------------------------------------------------------------------------------------
+struct Work {
+  size_t c_x = 0, c_xn = 0, c_qkv = 0, c_q = 0, c_k = 0, c_v = 0, c_att = 0, c_h = 0, c_gu = 0, c_part = 0;
+  float* x = nullptr;
+  char* xn = nullptr;
+  float* qkv = nullptr;
+  char *q = nullptr, *k = nullptr, *v = nullptr, *att = nullptr, *h = nullptr;
+  float* gu = nullptr;
+  float* part = nullptr;
+  int rows = 0;
+
+  sr_status ensure(const Model& m, int n) {
+    if (n <= rows) return SR_OK;
+    const size_t R = n, D = m.d.d_model, E = m.esz, F = m.d.ffn_dim;
+    const size_t HD = (size_t)m.d.n_heads * m.d.head_dim;
+    SR_TRY(grow(x, c_x, R * D));
+    SR_TRY(grow(xn, c_xn, R * D * E));
+    SR_TRY(grow(qkv, c_qkv, R * m.qkv_dim()));
+    SR_TRY(grow(q, c_q, R * HD * E));
+    SR_TRY(grow(k, c_k, R * m.kv_tok_elems() * E));
+    SR_TRY(grow(v, c_v, R * m.kv_tok_elems() * E));
+    SR_TRY(grow(att, c_att, R * HD * E));
+    SR_TRY(grow(h, c_h, R * F * E));
+    if (m.d.dtype == SR_DT_F32) SR_TRY(grow(gu, c_gu, R * F * (m.gated() ? 2 : 1)));
+    rows = n;
+    return SR_OK;
+  }
+  void release() {
+    void* ps[] = {x, xn, qkv, q, k, v, att, h, gu, part};
+    for (void* p : ps)
+      if (p) cudaFree(p);
+    *this = Work();
+  }
+};
+
+// Attention layout of one prefill call (packed sequences, optional shared prefix per layer).
+struct PrefillPlan {
+  const int* seq_off = nullptr;   // device [n_seq + 1]
+  int n_seq = 1;
+  const int* tile_seq = nullptr;  // device, bf16 path
+  const int* tile_q0 = nullptr;
+  int n_tiles = 0;
+  int pos0 = 0;
+  int n_pre = 0;
+  const char* pre_k = nullptr;    // per-layer prefix K / V stores: base + l * layer_stride
+  const char* pre_v = nullptr;
+  size_t pre_layer_bytes = 0;
+};
+// Where a prefill's per-layer K/V goes.
+struct PrefillKv {
+  char* store_k = nullptr;        // contiguous [rows][Hkv][dh] per layer at + l * store_layer_bytes
+  char* store_v = nullptr;
+  size_t store_layer_bytes = 0;
+  void* pool = nullptr;           // paged pool (layer 0 page 0) or nullptr
+  size_t pool_layer_bytes = 0;
+  const int* page_row = nullptr;  // page table row for positions (row_seq = null)
+};
+
+sr_status linear(const Model& m, const void* A, const void* W, void* C, int M, int N, int K, int epi,
+                 cudaStream_t st) {
+  if (m.d.dtype == SR_DT_BF16)
+    return gemm_bf16((const bf16*)A, (const bf16*)W, C, M, N, K, epi, st);
+  return gemm_f32((const float*)A, (const float*)W, (float*)C, M, N, K, epi, st);
+}
+
+// MLP block: x += W_down act(W_gate h, W_up h) (or GELU(W_fc h)), h = Norm(x) already in w.xn
+sr_status mlp(const Model& m, Work& w, const LayerW& lw, int M, cudaStream_t st) {
+  const int D = m.d.d_model, F = m.d.ffn_dim;
+  if (m.d.dtype == SR_DT_BF16) {
+    const int epi = m.d.act == SR_ACT_SWIGLU ? EPI_SWIGLU : (m.d.act == SR_ACT_GEGLU ? EPI_GEGLU : EPI_GELU);
+    SR_TRY(linear(m, w.xn, lw.wgu, w.h, M, m.gated() ? 2 * F : F, D, epi, st));
+  } else {
+    SR_TRY(linear(m, w.xn, lw.wgu, w.gu, M, m.gated() ? 2 * F : F, D, EPI_F32, st));
+    SR_TRY(launch_act(m.d.dtype, m.d.act, w.gu, M, F, w.h, st));
+  }
+  return linear(m, w.h, lw.wdown, w.x, M, D, F, EPI_ADD_F32, st);
+}
+
+// Prefill `M` rows (tokens / positions already on the device) through all layers; leaves the
+// residual stream in w.x.
+sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const int* pos, const PrefillPlan& plan,
+                          const PrefillKv& kv, cudaStream_t st) {
+  const sr_model_desc& d = m.d;
+  const int D = d.d_model, Hq = d.n_heads, Hkv = d.n_kv_heads, dh = d.head_dim;
+  SR_TRY(w.ensure(m, M));
+  SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, tok, pos, M, D, w.x, st));
+  for (int l = 0; l < d.n_layers; ++l) {
+    const LayerW& lw = m.L[l];
+    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, M, D, w.xn, st));
+    SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, M, m.qkv_dim(), D, EPI_F32, st));
+    char* kout = kv.store_k ? kv.store_k + l * kv.store_layer_bytes : w.k;
+    char* vout = kv.store_v ? kv.store_v + l * kv.store_layer_bytes : w.v;
+    KvSink sink{nullptr, nullptr, 0, nullptr};
+    if (kv.pool) sink = KvSink{static_cast<char*>(kv.pool) + l * kv.pool_layer_bytes, kv.page_row, 0, nullptr};
+    SR_TRY(launch_rope_store(d.dtype, w.qkv, M, pos, m.rope, Hq, Hkv, dh, w.q, kout, vout, sink, st));
+    const char* pk = plan.n_pre ? plan.pre_k + l * plan.pre_layer_bytes : nullptr;
+    const char* pv = plan.n_pre ? plan.pre_v + l * plan.pre_layer_bytes : nullptr;
+    if (d.dtype == SR_DT_BF16)
+      SR_TRY(launch_prefill_attention((const bf16*)w.q, (const bf16*)kout, (const bf16*)vout, (const bf16*)pk,
+                                      (const bf16*)pv, plan.n_pre, plan.seq_off, plan.n_seq, plan.tile_seq,
+                                      plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window, (bf16*)w.att,
+                                      st));
+    else
+      SR_TRY(launch_prefill_attention_f32((const float*)w.q, (const float*)kout, (const float*)vout,
+                                          (const float*)pk, (const float*)pv, plan.n_pre, plan.seq_off, plan.n_seq, M,
+                                          plan.pos0, Hq, Hkv, dh, d.window, (float*)w.att, st));
+    SR_TRY(linear(m, w.att, lw.wo, w.x, M, D, Hq * dh, EPI_ADD_F32, st));
+    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, M, D, w.xn, st));
+    SR_TRY(mlp(m, w, lw, M, st));
+  }
+  return SR_OK;
+}
+
+}  // namespace
+}  // namespace sr
+
+// =================================================================================================
+// context and batch state
+// =================================================================================================
+struct sr_ctx {
+  int device = 0;
+  cudaStream_t own = nullptr, st = nullptr;
+  sr::Model gen, rm;
+  sr::Work wg, wr;
+  // KV pool of the generator: [layer][page][2][Hkv][16][dh]; the last physical page is the
+  // prompt-tail template and never enters the free stack
+  size_t pool_bytes_req = 0;
+  char* pool = nullptr;
+  int pool_cap_pages = 0;  // physical pages including the template page
+  size_t page_elems = 0, page_bytes = 0;
+  // reward-model prompt KV store [layer][P][Hkv][dh] (K and V)
+  char *rm_pk = nullptr, *rm_pv = nullptr;
+  size_t c_rm_pk = 0, c_rm_pv = 0;
+  // candidate state
+  size_t c_len = 0, c_status = 0, c_tok = 0, c_pt = 0, c_live = 0, c_rset = 0, c_free = 0, c_tokin = 0, c_posin = 0,
+         c_kvlen = 0, c_tail = 0, c_prow = 0, c_ids = 0, c_reward = 0, c_rr = 0, c_logits = 0, c_mask = 0, c_prompt = 0,
+         c_iota = 0, c_meta = 0, c_hmeta = 0, c_out = 0, c_lastrow = 0, c_logits0 = 0;
+  int *len = nullptr, *status = nullptr, *tok = nullptr, *pt = nullptr, *live = nullptr, *rset = nullptr,
+      *free_stack = nullptr, *tok_in = nullptr, *pos_in = nullptr, *kv_len = nullptr, *tail_dst = nullptr,
+      *prompt_row = nullptr, *ids = nullptr, *prompt = nullptr, *iota = nullptr, *meta = nullptr, *out_tok = nullptr,
+      *last_row = nullptr;
+  float *reward = nullptr, *rr = nullptr, *logits = nullptr, *logits0 = nullptr;
+  uint8_t* mask = nullptr;
+  int* ctrl = nullptr;       // C_N ints
+  float* ctrlf = nullptr;    // 4 floats (r_cut, score)
+  int* h_ctrl = nullptr;     // pinned mirror
+  float* h_ctrlf = nullptr;
+  int* h_meta = nullptr;     // pinned staging for scoring plans
+  float* d_score = nullptr;
+  int* d_outlen = nullptr;
+};
+
+struct sr_batch {
+  int P = 0, N = 0, max_new = 0, eos_id = -1, n_sh = 0, has_tail = 0, max_pages = 0, n_pages = 0;
+  float temperature = 1.f, eos_bias = 0.f;
+  uint64_t seed = 0;
+  int n_live = 0, n_rset = 0, g = 0;  // g: tokens generated by every live candidate
+  bool active = false;
+};
+
+namespace sr {
+namespace {
+
+sr_status read_ctrl(sr_ctx* c) {
+  SR_CUDA(cudaMemcpyAsync(c->h_ctrl, c->ctrl, C_N * sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaMemcpyAsync(c->h_ctrlf, c->ctrlf, 4 * sizeof(float), cudaMemcpyDeviceToHost, c->st));
+  int* gerr = gemm_error_word();
+  if (gerr) SR_CUDA(cudaMemcpyAsync(c->h_ctrl + C_N, gerr, sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  if (gerr && c->h_ctrl[C_N] != 0)
+    return set_err(SR_ERR_TIMEOUT, "tensor-core GEMM wait expired (code %d)", c->h_ctrl[C_N]);
+  if (c->h_ctrl[C_ERR] == E_POOL_EMPTY) return set_err(SR_ERR_OOM, "KV page pool exhausted");
+  if (c->h_ctrl[C_ERR] == E_STATE) return set_err(SR_ERR_STATE, "no completed candidate");
+  return SR_OK;
+}
+
+size_t kv_bytes_per_token(const Model& m) { return (size_t)m.d.n_layers * 2 * m.kv_tok_elems() * m.esz; }
+
+int private_pages_full(int P, int max_new) { return (P + max_new - 2) / PAGE + 1 - P / PAGE; }
+
+// Size the pool for this call: the caller's byte budget, or everything that N candidates need.
+sr_status prepare_pool(sr_ctx* c, sr_batch& b) {
+  const Model& g = c->gen;
+  const size_t kvt = kv_bytes_per_token(g);
+  long long pages;
+  if (c->pool_bytes_req)
+    pages = (long long)(c->pool_bytes_req / (PAGE * kvt));
+  else
+    pages = b.P / PAGE + (long long)b.N * private_pages_full(b.P, b.max_new);
+  if (pages < 1) return set_err(SR_ERR_OOM, "KV pool smaller than one page");
+  if (pages > (1ll << 30)) return set_err(SR_ERR_INVALID_ARG, "KV pool too large");
+  b.n_pages = (int)pages;
+  c->page_elems = (size_t)2 * g.d.n_kv_heads * PAGE * g.d.head_dim;
+  c->page_bytes = c->page_elems * g.esz;
+  if (c->pool_cap_pages < b.n_pages + 1) {
+    if (c->pool) cudaFree(c->pool);
+    c->pool = nullptr;
+    c->pool_cap_pages = 0;
+    SR_CUDA(cudaMalloc(&c->pool, (size_t)(b.n_pages + 1) * c->page_bytes * g.d.n_layers));
+    c->pool_cap_pages = b.n_pages + 1;
+  }
+  return SR_OK;
+}
+
+size_t pool_layer_bytes(const sr_ctx* c) { return (size_t)c->pool_cap_pages * c->page_bytes; }
+
+sr_status prepare_state(sr_ctx* c, sr_batch& b) {
+  const size_t N = b.N;
+  SR_TRY(grow(c->len, c->c_len, N));
+  SR_TRY(grow(c->status, c->c_status, N));
+  SR_TRY(grow(c->tok, c->c_tok, N * b.max_new));
+  SR_TRY(grow(c->pt, c->c_pt, N * b.max_pages));
+  SR_TRY(grow(c->live, c->c_live, N));
+  SR_TRY(grow(c->rset, c->c_rset, N));
+  SR_TRY(grow(c->free_stack, c->c_free, (size_t)b.n_pages));
+  SR_TRY(grow(c->tok_in, c->c_tokin, N));
+  SR_TRY(grow(c->pos_in, c->c_posin, N));
+  SR_TRY(grow(c->kv_len, c->c_kvlen, N));
+  SR_TRY(grow(c->tail_dst, c->c_tail, N));
+  SR_TRY(grow(c->prompt_row, c->c_prow, (size_t)b.max_pages));
+  SR_TRY(grow(c->ids, c->c_ids, N));
+  SR_TRY(grow(c->reward, c->c_reward, N));
+  SR_TRY(grow(c->rr, c->c_rr, N));
+  SR_TRY(grow(c->mask, c->c_mask, N));
+  SR_TRY(grow(c->last_row, c->c_lastrow, N));
+  SR_TRY(grow(c->out_tok, c->c_out, (size_t)b.max_new));
+  SR_TRY(grow(c->logits, c->c_logits, N * c->gen.d.vocab));
+  SR_TRY(grow(c->logits0, c->c_logits0, (size_t)c->gen.d.vocab));
+  SR_TRY(c->wg.ensure(c->gen, std::max<int>(b.N, b.P)));
+  const int iota_n = std::max(c->gen.d.max_pos, c->rm.d.max_pos);
+  if (c->c_iota < (size_t)iota_n) {
+    std::vector<int> h(iota_n);
+    for (int i = 0; i < iota_n; ++i) h[i] = i;
+    SR_TRY(grow(c->iota, c->c_iota, (size_t)iota_n));
+    SR_CUDA(cudaMemcpy(c->iota, h.data(), iota_n * sizeof(int), cudaMemcpyHostToDevice));
+  }
+  SR_CUDA(cudaMemsetAsync(c->status, 0xff, N * sizeof(int), c->st));
+  SR_CUDA(cudaMemsetAsync(c->len, 0, N * sizeof(int), c->st));
+  SR_CUDA(cudaMemsetAsync(c->pt, 0, N * b.max_pages * sizeof(int), c->st));
+  return SR_OK;
+}
+
+// single-sequence prefill plan over [0, P): seq_off = {0, P}, tiles of 64 rows
+sr_status upload_single_plan(sr_ctx* c, int P, PrefillPlan& plan) {
+  const int n_tiles = (P + 63) / 64;
+  const size_t need = 2 + 2 * (size_t)n_tiles;
+  SR_TRY(grow_host(c->h_meta, c->c_hmeta, need));
+  SR_TRY(grow(c->meta, c->c_meta, need));
+  SR_CUDA(cudaStreamSynchronize(c->st));  // staging may still feed an earlier copy
+  c->h_meta[0] = 0;
+  c->h_meta[1] = P;
+  for (int t = 0; t < n_tiles; ++t) c->h_meta[2 + t] = 0, c->h_meta[2 + n_tiles + t] = t * 64;
+  SR_CUDA(cudaMemcpyAsync(c->meta, c->h_meta, need * sizeof(int), cudaMemcpyHostToDevice, c->st));
+  plan.seq_off = c->meta;
+  plan.n_seq = 1;
+  plan.tile_seq = c->meta + 2;
+  plan.tile_q0 = c->meta + 2 + n_tiles;
+  plan.n_tiles = n_tiles;
+  plan.pos0 = 0;
+  plan.n_pre = 0;
+  return SR_OK;
+}
+
+// Prompt through the reward model (KV kept for every later scoring chunk) and through the
+// generator (KV into the shared pages + tail template page; logits of the last position).
+sr_status prefill_prompt(sr_ctx* c, sr_batch& b) {
+  const Model& g = c->gen;
+  const Model& r = c->rm;
+  const int P = b.P;
+  // reward model
+  const size_t rm_layer = (size_t)P * r.kv_tok_elems() * r.esz;
+  SR_TRY(grow(c->rm_pk, c->c_rm_pk, rm_layer * r.d.n_layers));
+  SR_TRY(grow(c->rm_pv, c->c_rm_pv, rm_layer * r.d.n_layers));
+  PrefillPlan plan;
+  SR_TRY(upload_single_plan(c, P, plan));
+  PrefillKv kv;
+  kv.store_k = c->rm_pk;
+  kv.store_v = c->rm_pv;
+  kv.store_layer_bytes = rm_layer;
+  SR_TRY(forward_prefill(r, c->wr, P, c->prompt, c->iota, plan, kv, c->st));
+  // generator: pages for the prompt, KV into them
+  SR_TRY(ctl_prompt_pages(c->free_stack, c->ctrl, b.n_sh, b.has_tail, c->pool_cap_pages - 1, c->prompt_row, c->st));
+  PrefillKv gkv;
+  gkv.pool = c->pool;
+  gkv.pool_layer_bytes = pool_layer_bytes(c);
+  gkv.page_row = c->prompt_row;
+  SR_TRY(forward_prefill(g, c->wg, P, c->prompt, c->iota, plan, gkv, c->st));
+  // logits of the last prompt position (the distribution of token 0 of every candidate)
+  SR_TRY(launch_norm(g.d.dtype, g.d.norm, c->wg.x + (size_t)(P - 1) * g.d.d_model, g.final_w, g.final_b,
+                     g.d.norm_eps, 1, g.d.d_model, c->wg.xn, c->st));
+  SR_TRY(linear(g, c->wg.xn, g.lm_head, c->logits0, 1, g.d.vocab, g.d.d_model, EPI_F32, c->st));
+  return SR_OK;
+}
+
+// Admit candidates [start, start + count): pages, tail copy, token 0 from the prompt logits.
+sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
+  const Model& g = c->gen;
+  SR_TRY(ctl_admit(start, count, b.n_sh, b.has_tail, c->prompt_row, c->pt, b.max_pages, c->len, c->status, c->live,
+                   c->rset, c->free_stack, c->ctrl, c->tail_dst, c->st));
+  if (b.has_tail)
+    SR_TRY(launch_copy_page(g.d.dtype, c->pool, (long long)(pool_layer_bytes(c) / g.esz), g.d.n_layers,
+                            (int)c->page_elems, c->pool_cap_pages - 1, c->tail_dst, count, c->st));
+  SR_TRY(launch_sample(c->logits0, 0, count, g.d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias, b.eos_id,
+                       nullptr, c->tok, b.max_new, c->len, c->status, c->st));
+  SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack, c->st));
+  SR_TRY(read_ctrl(c));
+  b.n_live = c->h_ctrl[C_NLIVE];
+  b.n_rset = c->h_ctrl[C_NRSET];
+  b.g = 1;
+  return SR_OK;
+}
+
+// One batched decode step of every live candidate (positions P + g - 1), Eq. auto-regressive.
+sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
+  const Model& m = c->gen;
+  const sr_model_desc& d = m.d;
+  Work& w = c->wg;
+  const int n = b.n_live;
+  const int D = d.d_model, Hq = d.n_heads, Hkv = d.n_kv_heads, dh = d.head_dim;
+  SR_TRY(w.ensure(m, n));
+  SR_TRY(ctl_step_begin(b.P, c->live, c->ctrl, c->len, c->pt, b.max_pages, c->free_stack, c->tok, b.max_new,
+                        c->tok_in, c->pos_in, c->kv_len, c->st));
+  const int max_len = b.P + b.g;
+  const int splits = decode_attention_max_splits(std::min(max_len, d.window > 0 ? d.window : max_len));
+  if (splits > 1) SR_TRY(grow(w.part, w.c_part, decode_attention_part_floats(n, Hq, dh, splits)));
+  SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, c->tok_in, c->pos_in, n, D, w.x, c->st));
+  for (int l = 0; l < d.n_layers; ++l) {
+    const LayerW& lw = m.L[l];
+    char* pool_l = c->pool + l * pool_layer_bytes(c);
+    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, n, D, w.xn, c->st));
+    SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, n, m.qkv_dim(), D, EPI_F32, c->st));
+    SR_TRY(launch_rope_store(d.dtype, w.qkv, n, c->pos_in, m.rope, Hq, Hkv, dh, w.q, nullptr, nullptr,
+                             KvSink{pool_l, c->pt, b.max_pages, c->live}, c->st));
+    SR_TRY(launch_decode_attention(d.dtype, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
+                                   d.window, w.att, w.part, splits, c->st));
+    SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, c->st));
+    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, n, D, w.xn, c->st));
+    SR_TRY(mlp(m, w, lw, n, c->st));
+  }
+  SR_TRY(launch_norm(d.dtype, d.norm, w.x, m.final_w, m.final_b, d.norm_eps, n, D, w.xn, c->st));
+  SR_TRY(linear(m, w.xn, m.lm_head, c->logits, n, d.vocab, D, EPI_F32, c->st));
+  if (logits_host)
+    SR_CUDA(cudaMemcpyAsync(logits_host, c->logits, (size_t)n * d.vocab * sizeof(float), cudaMemcpyDeviceToHost,
+                            c->st));
+  SR_TRY(launch_sample(c->logits, d.vocab, n, d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias, b.eos_id,
+                       nullptr, c->tok, b.max_new, c->len, c->status, c->st));
+  SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack, c->st));
+  SR_TRY(read_ctrl(c));
+  b.n_live = c->h_ctrl[C_NLIVE];
+  b.g += 1;
+  return SR_OK;
+}
+
+__global__ void k_gather_rows(const int* __restrict__ ids, const int* __restrict__ off, const int* __restrict__ tok,
+                              int max_new, int P, int* tok_rows, int* pos_rows, int* last_row) {
+  const int j = blockIdx.x;
+  const int id = ids[j], r0 = off[j], n = off[j + 1] - off[j];
+  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+    tok_rows[r0 + i] = tok[(size_t)id * max_new + i];
+    pos_rows[r0 + i] = P + i;
+  }
+  if (threadIdx.x == 0) last_row[j] = r0 + n - 1;
+}
+
+constexpr int CHUNK_ROWS = 16384;  // reward-model rows (response tokens) per scoring pass
+
+// Rewards s(X ++ Y_k^{<= tau_k}) for candidates ids_h[0..n) with tau_k = taus[k] (Eq.
+// partial.reward.set); results into rewards_dev[0..n).  Each chunk runs the reward model over the
+// packed response tokens, attending to the prompt KV computed once at prefill.
+sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std::vector<int>& taus,
+                float* rewards_dev) {
+  const Model& r = c->rm;
+  const int n = (int)ids_h.size();
+  if (n == 0) return SR_OK;
+  const size_t rm_layer = (size_t)b.P * r.kv_tok_elems() * r.esz;
+  // plan chunks on the host: [ids | off | tiles_seq | tiles_q0] per chunk in one pinned buffer
+  struct Chunk {
+    int s0, ns, rows, n_tiles;
+    size_t meta;
+  };
+  std::vector<Chunk> chunks;
+  size_t meta_len = 0;
+  for (int s = 0; s < n;) {
+    Chunk ch{s, 0, 0, 0, meta_len};
+    while (s < n && (ch.ns == 0 || ch.rows + taus[s] <= CHUNK_ROWS)) {
+      ch.rows += taus[s];
+      ch.n_tiles += (taus[s] + 63) / 64;
+      ++ch.ns;
+      ++s;
+    }
+    meta_len += (size_t)ch.ns + (ch.ns + 1) + 2 * (size_t)ch.n_tiles;
+    chunks.push_back(ch);
+  }
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  SR_TRY(grow_host(c->h_meta, c->c_hmeta, meta_len));
+  SR_TRY(grow(c->meta, c->c_meta, meta_len));
+  int max_rows = 0;
+  for (const Chunk& ch : chunks) {
+    int* h = c->h_meta + ch.meta;
+    int* hid = h;
+    int* hoff = h + ch.ns;
+    int* hts = hoff + ch.ns + 1;
+    int* htq = hts + ch.n_tiles;
+    int o = 0, t = 0;
+    for (int j = 0; j < ch.ns; ++j) {
+      hid[j] = ids_h[ch.s0 + j];
+      hoff[j] = o;
+      const int tau = taus[ch.s0 + j];
+      for (int q0 = 0; q0 < tau; q0 += 64) hts[t] = j, htq[t] = q0, ++t;
+      o += tau;
+    }
+    hoff[ch.ns] = o;
+    max_rows = std::max(max_rows, ch.rows);
+  }
+  SR_CUDA(cudaMemcpyAsync(c->meta, c->h_meta, meta_len * sizeof(int), cudaMemcpyHostToDevice, c->st));
+  SR_TRY(c->wr.ensure(r, max_rows));
+  // token / position rows for the largest chunk
+  int *tok_rows = nullptr, *pos_rows = nullptr;
+  SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&tok_rows), (size_t)max_rows * sizeof(int), c->st));
+  SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&pos_rows), (size_t)max_rows * sizeof(int), c->st));
+  sr_status status = SR_OK;
+  for (const Chunk& ch : chunks) {
+    const int* did = c->meta + ch.meta;
+    const int* doff = did + ch.ns;
+    const int* dts = doff + ch.ns + 1;
+    const int* dtq = dts + ch.n_tiles;
+    k_gather_rows<<<ch.ns, 128, 0, c->st>>>(did, doff, c->tok, b.max_new, b.P, tok_rows, pos_rows, c->last_row);
+    if ((status = [&]() -> sr_status { SR_LAUNCH(); return SR_OK; }()) != SR_OK) break;
+    PrefillPlan plan;
+    plan.seq_off = doff;
+    plan.n_seq = ch.ns;
+    plan.tile_seq = dts;
+    plan.tile_q0 = dtq;
+    plan.n_tiles = ch.n_tiles;
+    plan.pos0 = b.P;
+    plan.n_pre = b.P;
+    plan.pre_k = c->rm_pk;
+    plan.pre_v = c->rm_pv;
+    plan.pre_layer_bytes = rm_layer;
+    if ((status = forward_prefill(r, c->wr, ch.rows, tok_rows, pos_rows, plan, PrefillKv(), c->st)) != SR_OK) break;
+    if ((status = launch_score_head(r.d.dtype, r.d.norm, c->wr.x, c->last_row, ch.ns, r.final_w, r.final_b,
+                                    r.d.norm_eps, r.score_head, r.d.d_model, rewards_dev + ch.s0, c->st)) != SR_OK)
+      break;
+  }
+  cudaFreeAsync(tok_rows, c->st);
+  cudaFreeAsync(pos_rows, c->st);
+  return status;
+}
+
+// ids and lengths of the round batch (host copies), plus their status
+sr_status read_rset(sr_ctx* c, sr_batch& b, std::vector<int>& ids, std::vector<int>& taus, std::vector<int>* st) {
+  ids.resize(b.n_rset);
+  taus.resize(b.n_rset);
+  std::vector<int> lens(b.N), stat(b.N);
+  SR_CUDA(cudaMemcpyAsync(ids.data(), c->rset, b.n_rset * sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaMemcpyAsync(lens.data(), c->len, b.N * sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaMemcpyAsync(stat.data(), c->status, b.N * sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  for (int i = 0; i < b.n_rset; ++i) taus[i] = lens[ids[i]];
+  if (st) {
+    st->resize(b.n_rset);
+    for (int i = 0; i < b.n_rset; ++i) (*st)[i] = stat[ids[i]];
+  }
+  return SR_OK;
+}
+
+sr_status validate_common(const sr_ctx* c, int P, int N, int max_new, float temperature, int eos_id) {
+  if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
+  if (P < 1 || N < 1 || N > MAX_BATCH || max_new < 1)
+    return set_err(SR_ERR_INVALID_ARG, "need P >= 1, 1 <= N <= %d, max_new >= 1", MAX_BATCH);
+  if (P + max_new > c->gen.d.max_pos || P + max_new > c->rm.d.max_pos)
+    return set_err(SR_ERR_INVALID_ARG, "P + max_new exceeds max_pos");
+  if (!(temperature > 0.f) || !std::isfinite(temperature)) return set_err(SR_ERR_INVALID_ARG, "temperature must be > 0");
+  if (eos_id < -1 || eos_id >= c->gen.d.vocab) return set_err(SR_ERR_INVALID_ARG, "eos_id out of range");
+  return SR_OK;
+}
+
+sr_status begin(sr_ctx* c, sr_batch& b, const int32_t* prompt, bool prompt_on_device, int P, int N, int max_new,
+                float temperature, float eos_bias, int eos_id, uint64_t seed) {
+  SR_TRY(validate_common(c, P, N, max_new, temperature, eos_id));
+  b = sr_batch();
+  b.P = P, b.N = N, b.max_new = max_new, b.temperature = temperature, b.eos_bias = eos_bias, b.eos_id = eos_id;
+  b.seed = seed;
+  b.n_sh = P / PAGE;
+  b.has_tail = P % PAGE != 0;
+  b.max_pages = (P + max_new - 1) / PAGE + 1;
+  SR_TRY(prepare_pool(c, b));
+  SR_TRY(prepare_state(c, b));
+  SR_TRY(grow(c->prompt, c->c_prompt, (size_t)P));
+  SR_CUDA(cudaMemcpyAsync(c->prompt, prompt, P * sizeof(int), prompt_on_device ? cudaMemcpyDeviceToDevice
+                                                                              : cudaMemcpyHostToDevice, c->st));
+  SR_TRY(ctl_pool_init(c->free_stack, b.n_pages, c->ctrl, c->st));
+  SR_TRY(prefill_prompt(c, b));
+  b.active = true;
+  return SR_OK;
+}
+
+// Algorithm 1 for a prepared batch; outputs stay on the device (c->out_tok, d_outlen, d_score).
+sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, sr_stats* st) {
+  const bool pool_mode = sched->kind == SR_SCHED_POOL_FULL;
+  std::vector<int> taus_sched(sched->tau, sched->tau + (sched->kind == SR_SCHED_FIXED ? sched->n_tau : 0));
+  sr_stats S;
+  memset(&S, 0, sizeof S);
+  S.pool_pages = b.n_pages;
+  double t0 = now_ms();
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  S.ms_prefill = now_ms() - t0;
+  // waves: alpha = 0 under a memory trigger is Best-of-N in pool-sized waves
+  std::vector<std::pair<int, int>> waves;
+  if (pool_mode && alpha == 0.f) {
+    SR_TRY(read_ctrl(c));
+    const int per = private_pages_full(b.P, b.max_new);
+    const int free_pages = c->h_ctrl[C_TOP];
+    const int w = per == 0 ? b.N : std::min(b.N, free_pages / per);
+    if (w <= 0) return set_err(SR_ERR_OOM, "KV pool cannot hold one candidate to max_new");
+    for (int s = 0; s < b.N; s += w) waves.push_back({s, std::min(w, b.N - s)});
+  } else {
+    waves.push_back({0, b.N});
+  }
+  S.waves = (int)waves.size();
+  std::vector<int> ids, taus, stat;
+  for (auto& wv : waves) {
+    double ta = now_ms();
+    SR_TRY(admit(c, b, wv.first, wv.second));
+    S.ms_decode += now_ms() - ta;
+    while (b.n_live > 0) {
+      const bool need = (b.P + b.g - 1) % PAGE == 0;
+      if (alpha > 0.f) {
+        bool trig;
+        if (pool_mode) {
+          trig = need && c->h_ctrl[C_TOP] < b.n_live;
+        } else {
+          trig = std::find(taus_sched.begin(), taus_sched.end(), b.g) != taus_sched.end();
+        }
+        if (trig) {
+          double ts = now_ms();
+          SR_TRY(read_rset(c, b, ids, taus, nullptr));
+          SR_TRY(score(c, b, ids, taus, c->rr));
+          SR_CUDA(cudaStreamSynchronize(c->st));
+          double tsel = now_ms();
+          S.ms_score += tsel - ts;
+          for (int t : taus) S.rm_tokens += t;
+          SR_TRY(ctl_round(b.P, b.n_sh, alpha, pool_mode && need ? 1 : 0, c->rr, c->rset, c->live, c->ctrl, c->ctrlf,
+                           c->status, c->len, c->reward, c->pt, b.max_pages, c->free_stack, nullptr, c->st));
+          SR_TRY(read_ctrl(c));
+          S.ms_select += now_ms() - tsel;
+          if (S.rounds < SR_MAX_ROUNDS) {
+            S.b_per_round[S.rounds] = b.n_rset;
+            S.step_per_round[S.rounds] = b.g;
+            S.k_per_round[S.rounds] = c->h_ctrl[C_K];
+            S.accepted_per_round[S.rounds] = c->h_ctrl[C_NACC];
+            S.r_cut_per_round[S.rounds] = c->h_ctrlf[0];
+          }
+          S.k_raised += c->h_ctrl[C_KRAISED];
+          S.rounds++;
+          b.n_live = c->h_ctrl[C_NLIVE];
+          b.n_rset = c->h_ctrl[C_NRSET];
+          if (b.n_live == 0) break;
+        }
+      }
+      if (need && c->h_ctrl[C_TOP] < b.n_live) return set_err(SR_ERR_OOM, "KV pool cannot hold the next decode step");
+      double td = now_ms();
+      SR_TRY(decode_step(c, b, nullptr));
+      S.ms_decode += now_ms() - td;
+      S.decode_steps++;
+    }
+    // completed candidates not scored in a round: final rewards
+    double tf = now_ms();
+    SR_TRY(read_rset(c, b, ids, taus, &stat));
+    std::vector<int> pid, ptau;
+    for (size_t i = 0; i < ids.size(); ++i)
+      if (stat[i] == ST_PENDING) pid.push_back(ids[i]), ptau.push_back(taus[i]);
+    if (!pid.empty()) {
+      SR_TRY(score(c, b, pid, ptau, c->rr));
+      SR_CUDA(cudaMemcpyAsync(c->ids, pid.data(), pid.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+      SR_TRY(ctl_mark_done(c->ids, c->rr, (int)pid.size(), c->status, c->reward, c->st));
+      SR_CUDA(cudaStreamSynchronize(c->st));
+      for (int t : ptau) S.rm_tokens += t;
+    }
+    S.ms_score += now_ms() - tf;
+  }
+  S.rm_tokens += b.P;
+  SR_TRY(ctl_final(b.N, c->status, c->reward, c->tok, b.max_new, c->len, c->out_tok, c->d_outlen, c->ctrlf + 1,
+                   c->ctrl, c->st));
+  SR_TRY(read_ctrl(c));
+  std::vector<int> lens(b.N), stv(b.N);
+  SR_CUDA(cudaMemcpy(lens.data(), c->len, b.N * sizeof(int), cudaMemcpyDeviceToHost));
+  SR_CUDA(cudaMemcpy(stv.data(), c->status, b.N * sizeof(int), cudaMemcpyDeviceToHost));
+  for (int i = 0; i < b.N; ++i) {
+    S.gen_tokens += lens[i];
+    S.n_completed += stv[i] == ST_DONE;
+  }
+  S.best_id = c->h_ctrl[C_BEST];
+  S.peak_pages_in_use = c->h_ctrl[C_PEAK];
+  S.ms_total = now_ms() - t0 + S.ms_prefill;
+  if (st) *st = S;
+  b.active = false;
+  return SR_OK;
+}
+
+}  // namespace
+}  // namespace sr
+
+using namespace sr;
+
+// =================================================================================================
+// C ABI
+// =================================================================================================
+extern "C" {
+
+const char* sr_last_error(void) { return g_msg.c_str(); }
+
+sr_status sr_init(sr_ctx** out, const sr_model_desc* gen, const void* gen_w, const sr_model_desc* rm,
+                  const void* rm_w, size_t kv_pool_bytes, int page_tokens, int device) {
+  if (!out) return set_err(SR_ERR_INVALID_ARG, "null output pointer");
+  *out = nullptr;
+  SR_TRY(check_desc(gen, "generator"));
+  SR_TRY(check_desc(rm, "reward model"));
+  if (!gen_w || !rm_w) return set_err(SR_ERR_INVALID_ARG, "null weights");
+  if (!gen->has_lm_head) return set_err(SR_ERR_INVALID_ARG, "generator needs an LM head");
+  if (!rm->has_scalar_head) return set_err(SR_ERR_INVALID_ARG, "reward model needs a scalar head");
+  if (gen->dtype != rm->dtype) return set_err(SR_ERR_INVALID_ARG, "generator and reward model dtypes differ");
+  if (gen->vocab != rm->vocab) return set_err(SR_ERR_INVALID_ARG, "generator and reward model vocabularies differ");
+  if (page_tokens != PAGE) return set_err(SR_ERR_INVALID_ARG, "page_tokens must be 16");
+  int ndev = 0;
+  SR_CUDA(cudaGetDeviceCount(&ndev));
+  if (device < 0 || device >= ndev) return set_err(SR_ERR_INVALID_ARG, "device %d not present", device);
+  SR_CUDA(cudaSetDevice(device));
+  sr_ctx* c = new sr_ctx();
+  c->device = device;
+  c->pool_bytes_req = kv_pool_bytes;
+  auto fail = [&](sr_status s) {
+    sr_destroy(c);
+    return s;
+  };
+  if (cudaStreamCreateWithFlags(&c->own, cudaStreamNonBlocking) != cudaSuccess)
+    return fail(set_err(SR_ERR_CUDA, "stream creation failed"));
+  c->st = c->own;
+  sr_status s;
+  if ((s = load_model(c->gen, gen, gen_w)) != SR_OK) return fail(s);
+  if ((s = load_model(c->rm, rm, rm_w)) != SR_OK) return fail(s);
+  if (cudaMalloc(&c->ctrl, C_N * sizeof(int)) != cudaSuccess || cudaMalloc(&c->ctrlf, 4 * sizeof(float)) ||
+      cudaMallocHost(&c->h_ctrl, (C_N + 1) * sizeof(int)) || cudaMallocHost(&c->h_ctrlf, 4 * sizeof(float)) ||
+      cudaMalloc(&c->d_score, sizeof(float)) || cudaMalloc(&c->d_outlen, sizeof(int)))
+    return fail(set_err(SR_ERR_OOM, "control buffers"));
+  cudaMemset(c->ctrl, 0, C_N * sizeof(int));
+  *out = c;
+  return SR_OK;
+}
+
+void sr_destroy(sr_ctx* c) {
+  if (!c) return;
+  cudaSetDevice(c->device);
+  if (c->st) cudaStreamSynchronize(c->st);
+  free_model(c->gen);
+  free_model(c->rm);
+  c->wg.release();
+  c->wr.release();
+  void* dev[] = {c->pool, c->rm_pk, c->rm_pv, c->len, c->status, c->tok, c->pt, c->live, c->rset, c->free_stack,
+                 c->tok_in, c->pos_in, c->kv_len, c->tail_dst, c->prompt_row, c->ids, c->prompt, c->iota, c->meta,
+                 c->out_tok, c->last_row, c->reward, c->rr, c->logits, c->logits0, c->mask, c->ctrl, c->ctrlf, c->d_score,
+                 c->d_outlen};
+  for (void* p : dev)
+    if (p) cudaFree(p);
+  if (c->h_ctrl) cudaFreeHost(c->h_ctrl);
+  if (c->h_ctrlf) cudaFreeHost(c->h_ctrlf);
+  if (c->h_meta) cudaFreeHost(c->h_meta);
+  if (c->own) cudaStreamDestroy(c->own);
+  delete c;
+}
+
+sr_status sr_set_stream(sr_ctx* c, void* stream) {
+  if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
+  c->st = stream ? static_cast<cudaStream_t>(stream) : c->own;
+  return SR_OK;
+}
+
+static sr_status check_sched(const sr_schedule* sched, float alpha) {
+  if (!sched) return set_err(SR_ERR_INVALID_ARG, "null schedule");
+  if (!(alpha >= 0.f && alpha <= 1.f)) return set_err(SR_ERR_INVALID_ARG, "alpha must be in [0, 1]");
+  if (sched->kind == SR_SCHED_FIXED) {
+    if (sched->n_tau < 0 || (sched->n_tau > 0 && !sched->tau)) return set_err(SR_ERR_INVALID_ARG, "bad tau list");
+    for (int i = 0; i < sched->n_tau; ++i)
+      if (sched->tau[i] < 1 || (i && sched->tau[i] <= sched->tau[i - 1]))
+        return set_err(SR_ERR_INVALID_ARG, "tau values must be ascending and >= 1");
+  } else if (sched->kind != SR_SCHED_POOL_FULL) {
+    return set_err(SR_ERR_INVALID_ARG, "unknown schedule kind");
+  }
+  return SR_OK;
+}
+
+static sr_status generate_impl(sr_ctx* c, const int32_t* prompt, bool dev, int P, int N, float alpha,
+                               const sr_schedule* sched, int max_new, float temperature, float eos_bias, int eos_id,
+                               uint64_t seed, sr_stats* st) {
+  SR_TRY(check_sched(sched, alpha));
+  SR_CUDA(cudaSetDevice(c->device));
+  sr_batch b;
+  SR_TRY(begin(c, b, prompt, dev, P, N, max_new, temperature, eos_bias, eos_id, seed));
+  return run_sr(c, b, alpha, sched, st);
+}
+
+sr_status sr_generate(sr_ctx* c, const int32_t* prompt, int P, int N, float alpha, const sr_schedule* sched,
+                      int max_new, float temperature, float eos_bias, int eos_id, uint64_t seed, int32_t* out_tokens,
+                      int* out_len, float* out_score, sr_stats* st) {
+  if (!c || !prompt || !out_tokens || !out_len || !out_score) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  SR_TRY(generate_impl(c, prompt, false, P, N, alpha, sched, max_new, temperature, eos_bias, eos_id, seed, st));
+  int L = 0;
+  SR_CUDA(cudaMemcpyAsync(&L, c->d_outlen, sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaMemcpyAsync(out_score, c->ctrlf + 1, sizeof(float), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  SR_CUDA(cudaMemcpyAsync(out_tokens, c->out_tok, L * sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  *out_len = L;
+  return SR_OK;
+}
+
+sr_status sr_generate_dev(sr_ctx* c, const int32_t* prompt_dev, int P, int N, float alpha, const sr_schedule* sched,
+                          int max_new, float temperature, float eos_bias, int eos_id, uint64_t seed,
+                          int32_t* out_tokens_dev, int* out_len_dev, float* out_score_dev, sr_stats* st,
+                          void* stream) {
+  if (!c || !prompt_dev || !out_tokens_dev || !out_len_dev || !out_score_dev)
+    return set_err(SR_ERR_INVALID_ARG, "null argument");
+  cudaStream_t prev = c->st;
+  if (stream) c->st = static_cast<cudaStream_t>(stream);
+  sr_status s = generate_impl(c, prompt_dev, true, P, N, alpha, sched, max_new, temperature, eos_bias, eos_id, seed, st);
+  if (s == SR_OK) {
+    cudaMemcpyAsync(out_tokens_dev, c->out_tok, (size_t)max_new * sizeof(int), cudaMemcpyDeviceToDevice, c->st);
+    cudaMemcpyAsync(out_len_dev, c->d_outlen, sizeof(int), cudaMemcpyDeviceToDevice, c->st);
+    cudaMemcpyAsync(out_score_dev, c->ctrlf + 1, sizeof(float), cudaMemcpyDeviceToDevice, c->st);
+    if (cudaStreamSynchronize(c->st) != cudaSuccess) s = set_err(SR_ERR_CUDA, "output copy failed");
+  }
+  c->st = prev;
+  return s;
+}
+
+// ---- component calls ----
+sr_status sr_batch_begin(sr_ctx* c, const int32_t* prompt, int P, int N, int max_new, float temperature,
+                         float eos_bias, int eos_id, uint64_t seed, sr_batch** out) {
+  if (!c || !prompt || !out) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  SR_CUDA(cudaSetDevice(c->device));
+  sr_batch* b = new sr_batch();
+  sr_status s = begin(c, *b, prompt, false, P, N, max_new, temperature, eos_bias, eos_id, seed);
+  if (s == SR_OK) s = admit(c, *b, 0, N);
+  if (s != SR_OK) {
+    delete b;
+    return s;
+  }
+  *out = b;
+  return SR_OK;
+}
+
+sr_status sr_decode_step(sr_ctx* c, sr_batch* b, float* logits_out) {
+  if (!c || !b) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  if (!b->active || b->n_live == 0) return set_err(SR_ERR_STATE, "no live candidate");
+  const bool need = (b->P + b->g - 1) % PAGE == 0;
+  if (need && c->h_ctrl[C_TOP] < b->n_live) return set_err(SR_ERR_OOM, "KV pool cannot hold the next decode step");
+  return decode_step(c, *b, logits_out);
+}
+
+sr_status sr_score_partial(sr_ctx* c, sr_batch* b, float* rewards, int* b_out) {
+  if (!c || !b || !rewards) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  if (!b->active) return set_err(SR_ERR_STATE, "batch not active");
+  std::vector<int> ids, taus;
+  SR_TRY(read_rset(c, *b, ids, taus, nullptr));
+  SR_TRY(score(c, *b, ids, taus, c->rr));
+  SR_CUDA(cudaMemcpyAsync(rewards, c->rr, ids.size() * sizeof(float), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaStreamSynchronize(c->st));
+  if (b_out) *b_out = (int)ids.size();
+  return SR_OK;
+}
+
+sr_status sr_reject_compact(sr_ctx* c, sr_batch* b, const float* rewards, float alpha, float* r_cut_out,
+                            int32_t* accepted_ids_out, int* b_out, int* b_live_out) {
+  if (!c || !b || !rewards) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  if (!b->active || b->n_rset == 0) return set_err(SR_ERR_STATE, "empty round batch");
+  if (!(alpha >= 0.f && alpha <= 1.f)) return set_err(SR_ERR_INVALID_ARG, "alpha must be in [0, 1]");
+  std::vector<int> ids(b->n_rset);
+  SR_CUDA(cudaMemcpyAsync(ids.data(), c->rset, b->n_rset * sizeof(int), cudaMemcpyDeviceToHost, c->st));
+  SR_CUDA(cudaMemcpyAsync(c->rr, rewards, b->n_rset * sizeof(float), cudaMemcpyHostToDevice, c->st));
+  SR_TRY(ctl_round(b->P, b->n_sh, alpha, 0, c->rr, c->rset, c->live, c->ctrl, c->ctrlf, c->status, c->len, c->reward,
+                   c->pt, b->max_pages, c->free_stack, c->mask, c->st));
+  std::vector<uint8_t> mask(b->n_rset);
+  SR_CUDA(cudaMemcpyAsync(mask.data(), c->mask, b->n_rset, cudaMemcpyDeviceToHost, c->st));
+  SR_TRY(read_ctrl(c));
+  int na = 0;
+  for (int i = 0; i < b->n_rset; ++i)
+    if (mask[i]) {
+      if (accepted_ids_out) accepted_ids_out[na] = ids[i];
+      ++na;
+    }
+  if (r_cut_out) *r_cut_out = c->h_ctrlf[0];
+  if (b_out) *b_out = na;
+  b->n_live = c->h_ctrl[C_NLIVE];
+  b->n_rset = c->h_ctrl[C_NRSET];
+  if (b_live_out) *b_live_out = b->n_live;
+  return SR_OK;
+}
+
+sr_status sr_batch_query(sr_ctx* c, const sr_batch* b, int32_t* ids_live, int32_t* lengths, int32_t* status,
+                         int32_t* tokens, int32_t* page_table, int32_t* free_stack, int* n_live, int* free_top,
+                         int* max_pages) {
+  if (!c || !b) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  SR_TRY(read_ctrl(c));
+  const size_t N = b->N;
+  if (ids_live) SR_CUDA(cudaMemcpy(ids_live, c->live, b->n_live * sizeof(int), cudaMemcpyDeviceToHost));
+  if (lengths) SR_CUDA(cudaMemcpy(lengths, c->len, N * sizeof(int), cudaMemcpyDeviceToHost));
+  if (status) SR_CUDA(cudaMemcpy(status, c->status, N * sizeof(int), cudaMemcpyDeviceToHost));
+  if (tokens) SR_CUDA(cudaMemcpy(tokens, c->tok, N * b->max_new * sizeof(int), cudaMemcpyDeviceToHost));
+  if (page_table) SR_CUDA(cudaMemcpy(page_table, c->pt, N * b->max_pages * sizeof(int), cudaMemcpyDeviceToHost));
+  if (free_stack) SR_CUDA(cudaMemcpy(free_stack, c->free_stack, c->h_ctrl[C_TOP] * sizeof(int), cudaMemcpyDeviceToHost));
+  if (n_live) *n_live = c->h_ctrl[C_NLIVE];
+  if (free_top) *free_top = c->h_ctrl[C_TOP];
+  if (max_pages) *max_pages = b->max_pages;
+  return SR_OK;
+}
+
+void sr_batch_end(sr_ctx* c, sr_batch* b) {
+  (void)c;
+  delete b;
+}
+
+// ---- kernel-level entry points ----
+sr_status sr_k_sample(const float* logits, long long ld, int b, int vocab, const int32_t* orig_ids,
+                      const int32_t* steps, uint64_t seed, float temperature, float eos_bias, int eos_id,
+                      int32_t* tokens_out, void* stream) {
+  if (!logits || !orig_ids || !steps || !tokens_out || b < 0 || vocab < 1)
+    return set_err(SR_ERR_INVALID_ARG, "sr_k_sample: bad argument");
+  return launch_sample(logits, ld, b, vocab, orig_ids, steps, seed, temperature, eos_bias, eos_id, tokens_out,
+                       nullptr, 0, nullptr, nullptr, static_cast<cudaStream_t>(stream));
+}
+
+sr_status sr_k_rcut(const float* rewards, int b, float alpha, int k_override, float* r_cut_out, uint8_t* mask_out,
+                    void* stream) {
+  if (!rewards || !r_cut_out || !mask_out) return set_err(SR_ERR_INVALID_ARG, "sr_k_rcut: null argument");
+  if (!(alpha >= 0.f && alpha <= 1.f)) return set_err(SR_ERR_INVALID_ARG, "alpha must be in [0, 1]");
+  return launch_rcut(rewards, b, alpha, k_override, r_cut_out, mask_out, static_cast<cudaStream_t>(stream));
+}
+
+sr_status sr_k_gemm(int dtype, const void* A, const void* W, void* C, int M, int N, int K, int epilogue,
+                    void* stream) {
+  if (!A || !W || !C) return set_err(SR_ERR_INVALID_ARG, "sr_k_gemm: null argument");
+  if (epilogue < 0 || epilogue > EPI_GELU) return set_err(SR_ERR_INVALID_ARG, "sr_k_gemm: bad epilogue");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (dtype == SR_DT_BF16) return gemm_bf16((const bf16*)A, (const bf16*)W, C, M, N, K, epilogue, st);
+  if (dtype == SR_DT_F32) return gemm_f32((const float*)A, (const float*)W, (float*)C, M, N, K, epilogue, st);
+  return set_err(SR_ERR_INVALID_ARG, "sr_k_gemm: bad dtype");
+}
+
+sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, const int32_t* page_table, int pt_stride,
+                                const int32_t* orig_ids, const int32_t* lens, int b, int n_heads, int n_kv_heads,
+                                int head_dim, int window, void* out, void* stream) {
+  if (!q || !pool || !page_table || !orig_ids || !lens || !out) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  if (b < 0 || n_kv_heads < 1 || n_heads < 1 || head_dim < 1) return set_err(SR_ERR_INVALID_ARG, "bad shape");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // partials for sequences longer than one split: sized for the longest possible context
+  std::vector<int> h(b);
+  if (b) SR_CUDA(cudaMemcpy(h.data(), lens, b * sizeof(int), cudaMemcpyDeviceToHost));
+  int mx = 1;
+  for (int x : h) mx = std::max(mx, x);
+  const int splits = decode_attention_max_splits(window > 0 ? std::min(mx, window) : mx);
+  float* part = nullptr;
+  if (splits > 1) SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&part),
+                                          decode_attention_part_floats(b, n_heads, head_dim, splits) * sizeof(float), st));
+  sr_status s = launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
+                                        head_dim, window, out, part, splits, st);
+  if (part) cudaFreeAsync(part, st);
+  return s;
+}
+
+sr_status sr_k_prefill_attention(const void* q, const void* k, const void* v, const void* k_pre, const void* v_pre,
+                                 int n_pre, const int32_t* seq_off, int n_seq, int pos0, int n_heads, int n_kv_heads,
+                                 int head_dim, int window, void* out, void* stream) {
+  if (!q || !k || !v || !seq_off || !out || n_seq < 1) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  if (n_pre > 0 && (!k_pre || !v_pre)) return set_err(SR_ERR_INVALID_ARG, "prefix pointers missing");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  std::vector<int> off(n_seq + 1);
+  SR_CUDA(cudaMemcpy(off.data(), seq_off, (n_seq + 1) * sizeof(int), cudaMemcpyDeviceToHost));
+  std::vector<int> ts, tq;
+  for (int j = 0; j < n_seq; ++j)
+    for (int q0 = 0; q0 < off[j + 1] - off[j]; q0 += 64) ts.push_back(j), tq.push_back(q0);
+  const int nt = (int)ts.size();
+  if (nt == 0) return SR_OK;
+  int* d = nullptr;
+  SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&d), 2 * nt * sizeof(int), st));
+  std::vector<int> hcat(ts);
+  hcat.insert(hcat.end(), tq.begin(), tq.end());
+  SR_CUDA(cudaMemcpyAsync(d, hcat.data(), 2 * nt * sizeof(int), cudaMemcpyHostToDevice, st));
+  sr_status s = launch_prefill_attention((const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)k_pre,
+                                         (const bf16*)v_pre, n_pre, seq_off, n_seq, d, d + nt, nt, pos0, n_heads,
+                                         n_kv_heads, head_dim, window, (bf16*)out, st);
+  cudaStreamSynchronize(st);  // the host copy of the tile list must outlive the upload
+  cudaFreeAsync(d, st);
+  return s;
+}
+
+}  // extern "C"

@@ -1,0 +1,53 @@
+"""The C-ABI library builds, loads and exports every entry point include/sr.h declares (CPU only)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+LIB = os.path.join(ROOT, "paper_2410_20290_gb300", "libsr.so")
+
+
+@pytest.fixture(scope="module")
+def lib_path():
+    if not os.path.exists(LIB):
+        from paper_2410_20290_gb300 import build
+        build.build()
+    return LIB
+
+
+def test_exports_every_declared_symbol(lib_path):
+    header = open(os.path.join(ROOT, "include", "sr.h")).read()
+    declared = set(re.findall(r"\b(sr_[a-z_0-9]+)\s*\(", header))
+    assert {"sr_init", "sr_generate", "sr_decode_step", "sr_score_partial", "sr_reject_compact"} <= declared
+    lib = ctypes.CDLL(lib_path)
+    missing = [s for s in sorted(declared) if not hasattr(lib, s)]
+    assert not missing, missing
+    nm = subprocess.run(["nm", "-D", "--defined-only", lib_path], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (sr_[a-z_0-9]+)$", nm, re.M))
+    assert declared <= exported
+
+
+def test_binding_names_match_header(lib_path):
+    from paper_2410_20290_gb300 import binding
+    for name in binding.declared_symbols():
+        if name == "sr_last_error":
+            continue
+        assert hasattr(binding, name), name
+
+
+def test_errors_without_device(lib_path):
+    """Argument checks run before any device work and report through sr_last_error."""
+    from paper_2410_20290_gb300 import binding as b
+    import sr_inputs as si
+    m = si.WORKLOADS["tiny"].gen
+    with pytest.raises(b.SrError) as e:
+        b.sr_init(m, None, m.replace(has_lm_head=0, has_scalar_head=1), None)
+    assert e.value.status == b.SR_ERR_INVALID_ARG
+    import numpy as np
+    x = np.zeros(4, np.float32)
+    with pytest.raises(b.SrError) as e:
+        b.sr_init(m.replace(n_heads=3, n_kv_heads=2), x, m.replace(has_lm_head=0, has_scalar_head=1), x)
+    assert e.value.status in (b.SR_ERR_UNSUPPORTED, b.SR_ERR_INVALID_ARG)
