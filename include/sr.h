@@ -87,6 +87,19 @@ typedef struct {
   const int* tau; /* host array, n_tau ascending values >= 1 */
 } sr_schedule;
 
+/* Kernel classes timed when profiling is on (sr_set_profiling). */
+enum {
+  SR_KC_GEMM_DECODE = 0,  /* generator projections + LM head during decode (tcgen05 / fp32 GEMM) */
+  SR_KC_GEMM_SCORE = 1,   /* reward-model projections while scoring partial / final responses */
+  SR_KC_GEMM_PROMPT = 2,  /* prompt prefill projections (both models) */
+  SR_KC_ATTN_DECODE = 3,  /* paged GQA decode attention (+ split combine) */
+  SR_KC_ATTN_PREFILL = 4, /* prefill attention (prompt and scoring) */
+  SR_KC_SAMPLE = 5,       /* Gumbel-max sampling */
+  SR_KC_ELEMENTWISE = 6,  /* embedding, norms, RoPE + KV append, activations, score head, page copies */
+  SR_KC_CONTROL = 7,      /* page allocation / release, rejection round, compaction, final argmax */
+  SR_KC_N = 8
+};
+
 #define SR_MAX_ROUNDS 64
 /* Per-call statistics of sr_generate (host struct filled by the library). */
 typedef struct {
@@ -105,7 +118,15 @@ typedef struct {
   long long decode_steps;                 /* batched decode steps */
   int pool_pages;                         /* pages in the KV pool */
   int peak_pages_in_use;
-  double ms_prefill, ms_decode, ms_score, ms_select, ms_total; /* device-timed phases */
+  double ms_prefill, ms_decode, ms_score, ms_select, ms_total; /* wall-clock phases, stream-synchronised */
+  /* per kernel class (zero unless profiling is on): summed CUDA-event time of the launches on the
+     context's stream, launch count, and the algorithmic work of those launches -- 2 M N K flops for
+     a GEMM, 4 dh (keys) flops per query head for attention; bytes = operands read + results
+     written once (decode attention: the shared prompt KV once plus each candidate's own KV) */
+  double kern_ms[SR_KC_N];
+  long long kern_launches[SR_KC_N];
+  double kern_flops[SR_KC_N];
+  double kern_bytes[SR_KC_N];
 } sr_stats;
 
 typedef struct sr_ctx sr_ctx;
@@ -114,7 +135,7 @@ typedef struct sr_batch sr_batch;
 /*
  * sr_init -- create a context on `device`.
  *   gen, gen_w : generator descriptor and weight blob (host or device pointer,
- *                detected with cudaPointerGetAttributes; copied, not retained).
+ *                copied with cudaMemcpyDefault under unified addressing; not retained).
  *                gen->has_lm_head must be 1.
  *   rm, rm_w   : reward-model descriptor and blob; rm->has_scalar_head must be 1.
  *                gen and rm must use the same vocabulary and dtype.
@@ -133,6 +154,8 @@ void sr_destroy(sr_ctx* ctx);
 const char* sr_last_error(void);
 /* Use `stream` (a cudaStream_t) for all later work of this context; NULL restores the context's stream. */
 sr_status sr_set_stream(sr_ctx* ctx, void* stream);
+/* Turn per-kernel-class CUDA-event timing on (1) or off (0); results land in sr_stats.kern_*. */
+sr_status sr_set_profiling(sr_ctx* ctx, int enable);
 
 /*
  * sr_generate -- Algorithm 1 end to end for one prompt (host buffers).

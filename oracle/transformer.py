@@ -26,6 +26,15 @@ softmax sums) accumulates in float64 before that rounding.  This keeps the
 oracle's results independent of how sequences are grouped into batches (a
 float32 BLAS call is not), which the exact Best-of-N pins rely on.
 
+Operand precision: with ``operand_rounding="bf16"`` the oracle rounds, to
+bfloat16 (round to nearest even), exactly the values a bf16 implementation
+feeds to its matrix units and keeps in its KV cache -- the normed inputs of
+every projection and of the LM head, q, k and v after RoPE, the attention
+output and the MLP hidden activation -- and nothing else; accumulation stays
+float64.  This states the arithmetic of "bf16 weights and operands, wide
+accumulation" so that a bf16 kernel can be held to a tight tolerance on
+rewards; the default (None) is the plain float32 forward.
+
 Two evaluation routes: ``forward`` recomputes a whole sequence with a causal
 mask; ``Decoder`` keeps a KV cache and appends one position per call.  Their
 agreement, and agreement of the pieces with torch's library routines, is
@@ -38,6 +47,13 @@ import numpy as np
 import sr_inputs as si
 
 F = np.float32
+
+
+def round_bf16(x):
+    """float32 -> nearest bfloat16 (ties to even), returned as float32."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
+    return r.astype(np.uint32).view(np.float32).reshape(np.shape(x))
 
 
 def mm(x, w64):
@@ -107,10 +123,12 @@ def attention(q, k, v, q_pos, k_pos, window):
 
 
 class Transformer:
-    def __init__(self, m: si.ModelDesc, weights: dict):
+    def __init__(self, m: si.ModelDesc, weights: dict, operand_rounding=None):
         self.m = m
         self.w = si.weights_as_f32(m, weights)
         self._w64 = {}
+        assert operand_rounding in (None, "bf16")
+        self.op = round_bf16 if operand_rounding == "bf16" else (lambda x: x)
 
     def W(self, name):
         """float64 copy of a weight matrix (cached) for float64-accumulated products."""
@@ -125,6 +143,10 @@ class Transformer:
             return rms_norm(x, self.w[prefix + "_w"], m.norm_eps)
         return layer_norm(x, self.w[prefix + "_w"], self.w[prefix + "_b"], m.norm_eps)
 
+    def norm_op(self, x, prefix):
+        """Norm whose output feeds a projection (an operand of the matrix units)."""
+        return self.op(self.norm(x, prefix))
+
     def embed(self, ids, positions):
         x = self.w["tok_emb"][np.asarray(ids)]
         if self.m.pos == si.POS_LEARNED:
@@ -133,7 +155,7 @@ class Transformer:
 
     def qkv(self, l, x, positions):
         m = self.m
-        h = self.norm(x, f"l{l}.attn_norm")
+        h = self.norm_op(x, f"l{l}.attn_norm")
         y = mm(h, self.W(f"l{l}.wqkv"))
         nq, nk = m.n_heads * m.head_dim, m.n_kv_heads * m.head_dim
         sh = x.shape[:-1]
@@ -143,28 +165,28 @@ class Transformer:
         if m.pos == si.POS_ROPE:
             q = apply_rope(q, positions, m.rope_theta)
             k = apply_rope(k, positions, m.rope_theta)
-        return q.astype(np.float32), k.astype(np.float32), v.astype(np.float32)
+        return self.op(q.astype(np.float32)), self.op(k.astype(np.float32)), self.op(v.astype(np.float32))
 
     def attn_out(self, l, x, a):
         sh = a.shape[:-2]
-        return (x + mm(a.reshape(*sh, -1), self.W(f"l{l}.wo"))).astype(np.float32)
+        return (x + mm(self.op(a.reshape(*sh, -1)), self.W(f"l{l}.wo"))).astype(np.float32)
 
     def mlp(self, l, x):
         m = self.m
-        h = self.norm(x, f"l{l}.mlp_norm")
+        h = self.norm_op(x, f"l{l}.mlp_norm")
         if m.act == si.ACT_SWIGLU:
             u = silu(mm(h, self.W(f"l{l}.w_gate"))) * mm(h, self.W(f"l{l}.w_up"))
         elif m.act == si.ACT_GEGLU:
             u = gelu_tanh(mm(h, self.W(f"l{l}.w_gate"))) * mm(h, self.W(f"l{l}.w_up"))
         else:
             u = gelu_tanh(mm(h, self.W(f"l{l}.w_fc")))
-        return (x + mm(u.astype(np.float32), self.W(f"l{l}.w_down"))).astype(np.float32)
+        return (x + mm(self.op(u.astype(np.float32)), self.W(f"l{l}.w_down"))).astype(np.float32)
 
     def final(self, x):
         return self.norm(x, "final_norm")
 
     def logits(self, hn):
-        return mm(hn, self.W("lm_head"))
+        return mm(self.op(hn), self.W("lm_head"))
 
     def score(self, hn):
         return (np.asarray(hn, np.float64) @ self.W("score_head")).astype(np.float32)

@@ -20,6 +20,9 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "sr.h")
 
 SR_OK, SR_ERR_INVALID_ARG, SR_ERR_OOM, SR_ERR_CUDA, SR_ERR_TIMEOUT, SR_ERR_STATE, SR_ERR_UNSUPPORTED = range(7)
 SR_MAX_ROUNDS = 64
+SR_KC_N = 8
+KERNEL_CLASSES = ("gemm_decode", "gemm_score", "gemm_prompt", "attn_decode", "attn_prefill", "sample", "elementwise",
+                  "control")
 
 
 class SrError(RuntimeError):
@@ -48,14 +51,19 @@ class sr_stats(ctypes.Structure):
                 ("gen_tokens", ctypes.c_longlong), ("rm_tokens", ctypes.c_longlong),
                 ("decode_steps", ctypes.c_longlong), ("pool_pages", ctypes.c_int),
                 ("peak_pages_in_use", ctypes.c_int), ("ms_prefill", ctypes.c_double), ("ms_decode", ctypes.c_double),
-                ("ms_score", ctypes.c_double), ("ms_select", ctypes.c_double), ("ms_total", ctypes.c_double)]
+                ("ms_score", ctypes.c_double), ("ms_select", ctypes.c_double), ("ms_total", ctypes.c_double),
+                ("kern_ms", ctypes.c_double * SR_KC_N), ("kern_launches", ctypes.c_longlong * SR_KC_N),
+                ("kern_flops", ctypes.c_double * SR_KC_N), ("kern_bytes", ctypes.c_double * SR_KC_N)]
 
     def as_dict(self) -> dict:
         r = self.rounds
         n = min(r, SR_MAX_ROUNDS)
-        out = {f: getattr(self, f) for f, _ in self._fields_ if not f.endswith("_round")}
+        out = {f: getattr(self, f) for f, _ in self._fields_ if not f.endswith("_round") and not f.startswith("kern_")}
         for f in ("b_per_round", "step_per_round", "k_per_round", "accepted_per_round", "r_cut_per_round"):
             out[f] = list(getattr(self, f))[:n]
+        out["kernels"] = {KERNEL_CLASSES[k]: dict(ms=self.kern_ms[k], launches=self.kern_launches[k],
+                                                  flops=self.kern_flops[k], bytes=self.kern_bytes[k])
+                          for k in range(SR_KC_N)}
         return out
 
 
@@ -67,6 +75,7 @@ _SIG = {
                 ctypes.c_size_t, _I, _I],
     "sr_destroy": [_P],
     "sr_set_stream": [_P, _P],
+    "sr_set_profiling": [_P, _I],
     "sr_generate": [_P, _P, _I, _I, _F, ctypes.POINTER(sr_schedule), _I, _F, _F, _I, ctypes.c_uint64, _P, _P, _P,
                     ctypes.POINTER(sr_stats)],
     "sr_generate_dev": [_P, _P, _I, _I, _F, ctypes.POINTER(sr_schedule), _I, _F, _F, _I, ctypes.c_uint64, _P, _P,
@@ -161,6 +170,10 @@ def sr_init(gen_desc, gen_w, rm_desc, rm_w, kv_pool_bytes: int = 0, page_tokens:
 
 def sr_destroy(ctx):
     LIB.sr_destroy(ctx)
+
+
+def sr_set_profiling(ctx, enable: bool = True):
+    _check(LIB.sr_set_profiling(ctx, int(bool(enable))))
 
 
 def sr_set_stream(ctx, stream=None):

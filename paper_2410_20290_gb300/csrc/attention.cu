@@ -182,9 +182,14 @@ __device__ __forceinline__ void mma16816(float* c, uint32_t a0, uint32_t a1, uin
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<uint32_t*>(&h);
+
+// (a, b) -> packed bf16 (hi) and the packed bf16 rounding of the remainders (lo)
+__device__ __forceinline__ void split_bf16(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  const float2 hf = __bfloat1622float2(h);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
 constexpr int BQ = 64, BKV = 64;
@@ -316,20 +321,24 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q
       o[i][0] *= corr[0], o[i][1] *= corr[0];
       o[i][2] *= corr[1], o[i][3] *= corr[1];
     }
-    // O += P V
+    // O += P V, with P carried as a bf16 hi + lo pair (P = hi + lo to ~16 mantissa bits) so the
+    // probabilities are not the coarsest operand in the product
 #pragma unroll
     for (int kk = 0; kk < BKV / 16; ++kk) {
-      const uint32_t a0 = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
-      const uint32_t a1 = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
-      const uint32_t a2 = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-      const uint32_t a3 = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+      uint32_t ah[4], al[4];
+      split_bf16(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+      split_bf16(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+      split_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+      split_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
 #pragma unroll
       for (int dp = 0; dp < DV / 16; ++dp) {
         uint32_t b0, b1, b2, b3;
         ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LDV + dp * 16 + (lane >> 4) * 8), b0,
                  b1, b2, b3);
-        mma16816(o[2 * dp], a0, a1, a2, a3, b0, b1);
-        mma16816(o[2 * dp + 1], a0, a1, a2, a3, b2, b3);
+        mma16816(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
+        mma16816(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+        mma16816(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
+        mma16816(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
       }
     }
   }

@@ -61,6 +61,78 @@ double now_ms() {
 }
 
 // -------------------------------------------------------------------------------------------------
+// per-kernel-class timing: CUDA events recorded on the launching stream around each launch,
+// read back after the stream synchronises
+// -------------------------------------------------------------------------------------------------
+struct Prof {
+  bool on = false;
+  std::vector<cudaEvent_t> ev;
+  size_t used = 0;
+  struct Rec {
+    int cls;
+    size_t a, b;
+    double fl, by;
+  };
+  std::vector<Rec> recs;
+  double ms[SR_KC_N] = {}, fl[SR_KC_N] = {}, by[SR_KC_N] = {};
+  long long n[SR_KC_N] = {};
+
+  cudaEvent_t take() {
+    if (used == ev.size()) {
+      cudaEvent_t e;
+      cudaEventCreate(&e);
+      ev.push_back(e);
+    }
+    return ev[used++];
+  }
+  long long begin(cudaStream_t st) {
+    if (!on) return -1;
+    const size_t i = used;
+    cudaEventRecord(take(), st);
+    return (long long)i;
+  }
+  void end(long long i, int cls, cudaStream_t st, double f, double b) {
+    if (i < 0) return;
+    const size_t j = used;
+    cudaEventRecord(take(), st);
+    recs.push_back({cls, (size_t)i, j, f, b});
+  }
+  void harvest() {  // every recorded event has completed (the stream was synchronised)
+    for (const Rec& r : recs) {
+      float t = 0.f;
+      if (cudaEventElapsedTime(&t, ev[r.a], ev[r.b]) == cudaSuccess) ms[r.cls] += t;
+      n[r.cls] += 1;
+      fl[r.cls] += r.fl;
+      by[r.cls] += r.by;
+    }
+    recs.clear();
+    used = 0;
+  }
+  void reset() {
+    recs.clear();
+    used = 0;
+    for (int c = 0; c < SR_KC_N; ++c) ms[c] = fl[c] = by[c] = 0, n[c] = 0;
+  }
+  ~Prof() {
+    for (cudaEvent_t e : ev) cudaEventDestroy(e);
+  }
+};
+
+// RAII timing scope for one launch (a no-op when profiling is off or pf is null)
+struct Scope {
+  Prof* p;
+  long long i;
+  int cls;
+  cudaStream_t st;
+  double f, b;
+  Scope(Prof* p_, int cls_, cudaStream_t st_, double f_ = 0, double b_ = 0)
+      : p(p_), i(p_ ? p_->begin(st_) : -1), cls(cls_), st(st_), f(f_), b(b_) {}
+  ~Scope() {
+    if (p) p->end(i, cls, st, f, b);
+  }
+};
+
+// -------------------------------------------------------------------------------------------------
 // model
 // -------------------------------------------------------------------------------------------------
 struct LayerW {
@@ -244,58 +316,90 @@ struct PrefillKv {
 };
 
 sr_status linear(const Model& m, const void* A, const void* W, void* C, int M, int N, int K, int epi,
-                 cudaStream_t st) {
+                 cudaStream_t st, Prof* pf = nullptr, int cls = SR_KC_GEMM_DECODE) {
+  const double E = m.esz;
+  const double out_b = (epi == EPI_F32) ? 4.0 * M * N : (epi == EPI_ADD_F32) ? 8.0 * M * N
+                       : (epi == EPI_SWIGLU || epi == EPI_GEGLU) ? E * M * N / 2 : E * M * N;
+  Scope sc(pf, cls, st, 2.0 * M * N * K, E * ((double)M * K + (double)N * K) + out_b);
   if (m.d.dtype == SR_DT_BF16)
     return gemm_bf16((const bf16*)A, (const bf16*)W, C, M, N, K, epi, st);
   return gemm_f32((const float*)A, (const float*)W, (float*)C, M, N, K, epi, st);
 }
 
 // MLP block: x += W_down act(W_gate h, W_up h) (or GELU(W_fc h)), h = Norm(x) already in w.xn
-sr_status mlp(const Model& m, Work& w, const LayerW& lw, int M, cudaStream_t st) {
+sr_status mlp(const Model& m, Work& w, const LayerW& lw, int M, cudaStream_t st, Prof* pf, int cls) {
   const int D = m.d.d_model, F = m.d.ffn_dim;
   if (m.d.dtype == SR_DT_BF16) {
     const int epi = m.d.act == SR_ACT_SWIGLU ? EPI_SWIGLU : (m.d.act == SR_ACT_GEGLU ? EPI_GEGLU : EPI_GELU);
-    SR_TRY(linear(m, w.xn, lw.wgu, w.h, M, m.gated() ? 2 * F : F, D, epi, st));
+    SR_TRY(linear(m, w.xn, lw.wgu, w.h, M, m.gated() ? 2 * F : F, D, epi, st, pf, cls));
   } else {
-    SR_TRY(linear(m, w.xn, lw.wgu, w.gu, M, m.gated() ? 2 * F : F, D, EPI_F32, st));
+    SR_TRY(linear(m, w.xn, lw.wgu, w.gu, M, m.gated() ? 2 * F : F, D, EPI_F32, st, pf, cls));
+    Scope sc(pf, SR_KC_ELEMENTWISE, st);
     SR_TRY(launch_act(m.d.dtype, m.d.act, w.gu, M, F, w.h, st));
   }
-  return linear(m, w.h, lw.wdown, w.x, M, D, F, EPI_ADD_F32, st);
+  return linear(m, w.h, lw.wdown, w.x, M, D, F, EPI_ADD_F32, st, pf, cls);
 }
 
 // Prefill `M` rows (tokens / positions already on the device) through all layers; leaves the
 // residual stream in w.x.
 sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const int* pos, const PrefillPlan& plan,
-                          const PrefillKv& kv, cudaStream_t st) {
+                          const PrefillKv& kv, cudaStream_t st, Prof* pf, int gcls, double attn_flops) {
   const sr_model_desc& d = m.d;
   const int D = d.d_model, Hq = d.n_heads, Hkv = d.n_kv_heads, dh = d.head_dim;
   SR_TRY(w.ensure(m, M));
-  SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, tok, pos, M, D, w.x, st));
+  {
+    Scope sc(pf, SR_KC_ELEMENTWISE, st);
+    SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, tok, pos, M, D, w.x, st));
+  }
   for (int l = 0; l < d.n_layers; ++l) {
     const LayerW& lw = m.L[l];
-    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, M, D, w.xn, st));
-    SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, M, m.qkv_dim(), D, EPI_F32, st));
+    {
+      Scope sc(pf, SR_KC_ELEMENTWISE, st);
+      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, M, D, w.xn, st));
+    }
+    SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, M, m.qkv_dim(), D, EPI_F32, st, pf, gcls));
     char* kout = kv.store_k ? kv.store_k + l * kv.store_layer_bytes : w.k;
     char* vout = kv.store_v ? kv.store_v + l * kv.store_layer_bytes : w.v;
     KvSink sink{nullptr, nullptr, 0, nullptr};
     if (kv.pool) sink = KvSink{static_cast<char*>(kv.pool) + l * kv.pool_layer_bytes, kv.page_row, 0, nullptr};
-    SR_TRY(launch_rope_store(d.dtype, w.qkv, M, pos, m.rope, Hq, Hkv, dh, w.q, kout, vout, sink, st));
+    {
+      Scope sc(pf, SR_KC_ELEMENTWISE, st);
+      SR_TRY(launch_rope_store(d.dtype, w.qkv, M, pos, m.rope, Hq, Hkv, dh, w.q, kout, vout, sink, st));
+    }
     const char* pk = plan.n_pre ? plan.pre_k + l * plan.pre_layer_bytes : nullptr;
     const char* pv = plan.n_pre ? plan.pre_v + l * plan.pre_layer_bytes : nullptr;
-    if (d.dtype == SR_DT_BF16)
-      SR_TRY(launch_prefill_attention((const bf16*)w.q, (const bf16*)kout, (const bf16*)vout, (const bf16*)pk,
-                                      (const bf16*)pv, plan.n_pre, plan.seq_off, plan.n_seq, plan.tile_seq,
-                                      plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window, (bf16*)w.att,
-                                      st));
-    else
-      SR_TRY(launch_prefill_attention_f32((const float*)w.q, (const float*)kout, (const float*)vout,
-                                          (const float*)pk, (const float*)pv, plan.n_pre, plan.seq_off, plan.n_seq, M,
-                                          plan.pos0, Hq, Hkv, dh, d.window, (float*)w.att, st));
-    SR_TRY(linear(m, w.att, lw.wo, w.x, M, D, Hq * dh, EPI_ADD_F32, st));
-    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, M, D, w.xn, st));
-    SR_TRY(mlp(m, w, lw, M, st));
+    const double kvb = (double)m.kv_tok_elems() * m.esz;
+    {
+      Scope sa(pf, SR_KC_ATTN_PREFILL, st, attn_flops,
+               2.0 * M * (double)Hq * dh * m.esz + 2.0 * kvb * (M + (double)plan.n_pre));
+      if (d.dtype == SR_DT_BF16)
+        SR_TRY(launch_prefill_attention((const bf16*)w.q, (const bf16*)kout, (const bf16*)vout, (const bf16*)pk,
+                                        (const bf16*)pv, plan.n_pre, plan.seq_off, plan.n_seq, plan.tile_seq,
+                                        plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window, (bf16*)w.att,
+                                        st));
+      else
+        SR_TRY(launch_prefill_attention_f32((const float*)w.q, (const float*)kout, (const float*)vout,
+                                            (const float*)pk, (const float*)pv, plan.n_pre, plan.seq_off, plan.n_seq,
+                                            M, plan.pos0, Hq, Hkv, dh, d.window, (float*)w.att, st));
+    }
+    SR_TRY(linear(m, w.att, lw.wo, w.x, M, D, Hq * dh, EPI_ADD_F32, st, pf, gcls));
+    {
+      Scope sc(pf, SR_KC_ELEMENTWISE, st);
+      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, M, D, w.xn, st));
+    }
+    SR_TRY(mlp(m, w, lw, M, st, pf, gcls));
   }
   return SR_OK;
+}
+
+// algorithmic flops of causal prefill attention: query i of a sequence sees n_pre + i + 1 keys
+double prefill_attn_flops(const Model& m, const std::vector<int>& taus, size_t s0, size_t n, int n_pre) {
+  double keys = 0;
+  for (size_t j = s0; j < s0 + n; ++j) {
+    const double t = taus[j];
+    keys += t * n_pre + t * (t + 1) / 2;
+  }
+  return 4.0 * m.d.n_heads * m.d.head_dim * keys;  // per layer
 }
 
 }  // namespace
@@ -335,6 +439,7 @@ struct sr_ctx {
   int* h_meta = nullptr;     // pinned staging for scoring plans
   float* d_score = nullptr;
   int* d_outlen = nullptr;
+  sr::Prof prof;
 };
 
 struct sr_batch {
@@ -356,6 +461,7 @@ sr_status read_ctrl(sr_ctx* c) {
   SR_CUDA(cudaStreamSynchronize(c->st));
   if (gerr && c->h_ctrl[C_N] != 0)
     return set_err(SR_ERR_TIMEOUT, "tensor-core GEMM wait expired (code %d)", c->h_ctrl[C_N]);
+  c->prof.harvest();
   if (c->h_ctrl[C_ERR] == E_POOL_EMPTY) return set_err(SR_ERR_OOM, "KV page pool exhausted");
   if (c->h_ctrl[C_ERR] == E_STATE) return set_err(SR_ERR_STATE, "no completed candidate");
   return SR_OK;
@@ -464,32 +570,57 @@ sr_status prefill_prompt(sr_ctx* c, sr_batch& b) {
   kv.store_k = c->rm_pk;
   kv.store_v = c->rm_pv;
   kv.store_layer_bytes = rm_layer;
-  SR_TRY(forward_prefill(r, c->wr, P, c->prompt, c->iota, plan, kv, c->st));
+  Prof* pf = &c->prof;
+  const std::vector<int> ptau(1, P);
+  SR_TRY(forward_prefill(r, c->wr, P, c->prompt, c->iota, plan, kv, c->st, pf, SR_KC_GEMM_PROMPT,
+                         prefill_attn_flops(r, ptau, 0, 1, 0)));
   // generator: pages for the prompt, KV into them
-  SR_TRY(ctl_prompt_pages(c->free_stack, c->ctrl, b.n_sh, b.has_tail, c->pool_cap_pages - 1, c->prompt_row, c->st));
+  {
+    Scope sc(pf, SR_KC_CONTROL, c->st);
+    SR_TRY(ctl_prompt_pages(c->free_stack, c->ctrl, b.n_sh, b.has_tail, c->pool_cap_pages - 1, c->prompt_row,
+                            c->st));
+  }
   PrefillKv gkv;
   gkv.pool = c->pool;
   gkv.pool_layer_bytes = pool_layer_bytes(c);
   gkv.page_row = c->prompt_row;
-  SR_TRY(forward_prefill(g, c->wg, P, c->prompt, c->iota, plan, gkv, c->st));
+  SR_TRY(forward_prefill(g, c->wg, P, c->prompt, c->iota, plan, gkv, c->st, pf, SR_KC_GEMM_PROMPT,
+                         prefill_attn_flops(g, ptau, 0, 1, 0)));
   // logits of the last prompt position (the distribution of token 0 of every candidate)
-  SR_TRY(launch_norm(g.d.dtype, g.d.norm, c->wg.x + (size_t)(P - 1) * g.d.d_model, g.final_w, g.final_b,
-                     g.d.norm_eps, 1, g.d.d_model, c->wg.xn, c->st));
-  SR_TRY(linear(g, c->wg.xn, g.lm_head, c->logits0, 1, g.d.vocab, g.d.d_model, EPI_F32, c->st));
+  {
+    Scope sc(pf, SR_KC_ELEMENTWISE, c->st);
+    SR_TRY(launch_norm(g.d.dtype, g.d.norm, c->wg.x + (size_t)(P - 1) * g.d.d_model, g.final_w, g.final_b,
+                       g.d.norm_eps, 1, g.d.d_model, c->wg.xn, c->st));
+  }
+  SR_TRY(linear(g, c->wg.xn, g.lm_head, c->logits0, 1, g.d.vocab, g.d.d_model, EPI_F32, c->st, pf,
+                SR_KC_GEMM_PROMPT));
   return SR_OK;
 }
 
 // Admit candidates [start, start + count): pages, tail copy, token 0 from the prompt logits.
 sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
   const Model& g = c->gen;
-  SR_TRY(ctl_admit(start, count, b.n_sh, b.has_tail, c->prompt_row, c->pt, b.max_pages, c->len, c->status, c->live,
-                   c->rset, c->free_stack, c->ctrl, c->tail_dst, c->st));
-  if (b.has_tail)
+  Prof* pf = &c->prof;
+  {
+    Scope sc(pf, SR_KC_CONTROL, c->st);
+    SR_TRY(ctl_admit(start, count, b.n_sh, b.has_tail, c->prompt_row, c->pt, b.max_pages, c->len, c->status,
+                     c->live, c->rset, c->free_stack, c->ctrl, c->tail_dst, c->st));
+  }
+  if (b.has_tail) {
+    Scope sc(pf, SR_KC_ELEMENTWISE, c->st);
     SR_TRY(launch_copy_page(g.d.dtype, c->pool, (long long)(pool_layer_bytes(c) / g.esz), g.d.n_layers,
                             (int)c->page_elems, c->pool_cap_pages - 1, c->tail_dst, count, c->st));
-  SR_TRY(launch_sample(c->logits0, 0, count, g.d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias, b.eos_id,
-                       nullptr, c->tok, b.max_new, c->len, c->status, c->st));
-  SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack, c->st));
+  }
+  {
+    Scope sc(pf, SR_KC_SAMPLE, c->st, 0, 4.0 * g.d.vocab);
+    SR_TRY(launch_sample(c->logits0, 0, count, g.d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias,
+                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, c->st));
+  }
+  {
+    Scope sc(pf, SR_KC_CONTROL, c->st);
+    SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack,
+                        c->st));
+  }
   SR_TRY(read_ctrl(c));
   b.n_live = c->h_ctrl[C_NLIVE];
   b.n_rset = c->h_ctrl[C_NRSET];
@@ -505,33 +636,69 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
   const int n = b.n_live;
   const int D = d.d_model, Hq = d.n_heads, Hkv = d.n_kv_heads, dh = d.head_dim;
   SR_TRY(w.ensure(m, n));
-  SR_TRY(ctl_step_begin(b.P, c->live, c->ctrl, c->len, c->pt, b.max_pages, c->free_stack, c->tok, b.max_new,
-                        c->tok_in, c->pos_in, c->kv_len, c->st));
+  Prof* pf = &c->prof;
+  cudaStream_t st = c->st;
+  {
+    Scope sc(pf, SR_KC_CONTROL, st);
+    SR_TRY(ctl_step_begin(b.P, c->live, c->ctrl, c->len, c->pt, b.max_pages, c->free_stack, c->tok, b.max_new,
+                          c->tok_in, c->pos_in, c->kv_len, st));
+  }
   const int max_len = b.P + b.g;
-  const int splits = decode_attention_max_splits(std::min(max_len, d.window > 0 ? d.window : max_len));
+  const int eff_len = d.window > 0 ? std::min(max_len, d.window) : max_len;
+  const int splits = decode_attention_max_splits(eff_len);
   if (splits > 1) SR_TRY(grow(w.part, w.c_part, decode_attention_part_floats(n, Hq, dh, splits)));
-  SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, c->tok_in, c->pos_in, n, D, w.x, c->st));
+  // algorithmic work of one decode-attention launch: the shared prompt KV once, each candidate's own KV,
+  // q in and the output out
+  const double kvb = 2.0 * Hkv * dh * m.esz;
+  const double shared = (eff_len == max_len) ? (double)PAGE * b.n_sh : 0.0;
+  const double attn_bytes = kvb * (shared + (double)n * (eff_len - shared)) + 2.0 * n * Hq * dh * m.esz;
+  const double attn_flops = 4.0 * n * Hq * dh * (double)eff_len;
+  {
+    Scope sc(pf, SR_KC_ELEMENTWISE, st);
+    SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, c->tok_in, c->pos_in, n, D, w.x, st));
+  }
   for (int l = 0; l < d.n_layers; ++l) {
     const LayerW& lw = m.L[l];
     char* pool_l = c->pool + l * pool_layer_bytes(c);
-    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, n, D, w.xn, c->st));
-    SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, n, m.qkv_dim(), D, EPI_F32, c->st));
-    SR_TRY(launch_rope_store(d.dtype, w.qkv, n, c->pos_in, m.rope, Hq, Hkv, dh, w.q, nullptr, nullptr,
-                             KvSink{pool_l, c->pt, b.max_pages, c->live}, c->st));
-    SR_TRY(launch_decode_attention(d.dtype, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
-                                   d.window, w.att, w.part, splits, c->st));
-    SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, c->st));
-    SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, n, D, w.xn, c->st));
-    SR_TRY(mlp(m, w, lw, n, c->st));
+    {
+      Scope sc(pf, SR_KC_ELEMENTWISE, st);
+      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, n, D, w.xn, st));
+    }
+    SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, n, m.qkv_dim(), D, EPI_F32, st, pf, SR_KC_GEMM_DECODE));
+    {
+      Scope sc(pf, SR_KC_ELEMENTWISE, st);
+      SR_TRY(launch_rope_store(d.dtype, w.qkv, n, c->pos_in, m.rope, Hq, Hkv, dh, w.q, nullptr, nullptr,
+                               KvSink{pool_l, c->pt, b.max_pages, c->live}, st));
+    }
+    {
+      Scope sc(pf, SR_KC_ATTN_DECODE, st, attn_flops, attn_bytes);
+      SR_TRY(launch_decode_attention(d.dtype, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
+                                     d.window, w.att, w.part, splits, st));
+    }
+    SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, st, pf, SR_KC_GEMM_DECODE));
+    {
+      Scope sc(pf, SR_KC_ELEMENTWISE, st);
+      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, n, D, w.xn, st));
+    }
+    SR_TRY(mlp(m, w, lw, n, st, pf, SR_KC_GEMM_DECODE));
   }
-  SR_TRY(launch_norm(d.dtype, d.norm, w.x, m.final_w, m.final_b, d.norm_eps, n, D, w.xn, c->st));
-  SR_TRY(linear(m, w.xn, m.lm_head, c->logits, n, d.vocab, D, EPI_F32, c->st));
+  {
+    Scope sc(pf, SR_KC_ELEMENTWISE, st);
+    SR_TRY(launch_norm(d.dtype, d.norm, w.x, m.final_w, m.final_b, d.norm_eps, n, D, w.xn, st));
+  }
+  SR_TRY(linear(m, w.xn, m.lm_head, c->logits, n, d.vocab, D, EPI_F32, st, pf, SR_KC_GEMM_DECODE));
   if (logits_host)
     SR_CUDA(cudaMemcpyAsync(logits_host, c->logits, (size_t)n * d.vocab * sizeof(float), cudaMemcpyDeviceToHost,
-                            c->st));
-  SR_TRY(launch_sample(c->logits, d.vocab, n, d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias, b.eos_id,
-                       nullptr, c->tok, b.max_new, c->len, c->status, c->st));
-  SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack, c->st));
+                            st));
+  {
+    Scope sc(pf, SR_KC_SAMPLE, st, 0, 4.0 * n * d.vocab);
+    SR_TRY(launch_sample(c->logits, d.vocab, n, d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias,
+                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, st));
+  }
+  {
+    Scope sc(pf, SR_KC_CONTROL, st);
+    SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack, st));
+  }
   SR_TRY(read_ctrl(c));
   b.n_live = c->h_ctrl[C_NLIVE];
   b.g += 1;
@@ -611,7 +778,10 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
     const int* doff = did + ch.ns;
     const int* dts = doff + ch.ns + 1;
     const int* dtq = dts + ch.n_tiles;
-    k_gather_rows<<<ch.ns, 128, 0, c->st>>>(did, doff, c->tok, b.max_new, b.P, tok_rows, pos_rows, c->last_row);
+    {
+      Scope sc(&c->prof, SR_KC_ELEMENTWISE, c->st);
+      k_gather_rows<<<ch.ns, 128, 0, c->st>>>(did, doff, c->tok, b.max_new, b.P, tok_rows, pos_rows, c->last_row);
+    }
     if ((status = [&]() -> sr_status { SR_LAUNCH(); return SR_OK; }()) != SR_OK) break;
     PrefillPlan plan;
     plan.seq_off = doff;
@@ -624,7 +794,10 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
     plan.pre_k = c->rm_pk;
     plan.pre_v = c->rm_pv;
     plan.pre_layer_bytes = rm_layer;
-    if ((status = forward_prefill(r, c->wr, ch.rows, tok_rows, pos_rows, plan, PrefillKv(), c->st)) != SR_OK) break;
+    if ((status = forward_prefill(r, c->wr, ch.rows, tok_rows, pos_rows, plan, PrefillKv(), c->st, &c->prof,
+                                  SR_KC_GEMM_SCORE, prefill_attn_flops(r, taus, ch.s0, ch.ns, b.P))) != SR_OK)
+      break;
+    Scope sc(&c->prof, SR_KC_ELEMENTWISE, c->st);
     if ((status = launch_score_head(r.d.dtype, r.d.norm, c->wr.x, c->last_row, ch.ns, r.final_w, r.final_b,
                                     r.d.norm_eps, r.score_head, r.d.d_model, rewards_dev + ch.s0, c->st)) != SR_OK)
       break;
@@ -665,6 +838,7 @@ sr_status validate_common(const sr_ctx* c, int P, int N, int max_new, float temp
 sr_status begin(sr_ctx* c, sr_batch& b, const int32_t* prompt, bool prompt_on_device, int P, int N, int max_new,
                 float temperature, float eos_bias, int eos_id, uint64_t seed) {
   SR_TRY(validate_common(c, P, N, max_new, temperature, eos_id));
+  c->prof.reset();
   b = sr_batch();
   b.P = P, b.N = N, b.max_new = max_new, b.temperature = temperature, b.eos_bias = eos_bias, b.eos_id = eos_id;
   b.seed = seed;
@@ -727,8 +901,12 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
           double tsel = now_ms();
           S.ms_score += tsel - ts;
           for (int t : taus) S.rm_tokens += t;
-          SR_TRY(ctl_round(b.P, b.n_sh, alpha, pool_mode && need ? 1 : 0, c->rr, c->rset, c->live, c->ctrl, c->ctrlf,
-                           c->status, c->len, c->reward, c->pt, b.max_pages, c->free_stack, nullptr, c->st));
+          {
+            Scope sc(&c->prof, SR_KC_CONTROL, c->st);
+            SR_TRY(ctl_round(b.P, b.n_sh, alpha, pool_mode && need ? 1 : 0, c->rr, c->rset, c->live, c->ctrl,
+                             c->ctrlf, c->status, c->len, c->reward, c->pt, b.max_pages, c->free_stack, nullptr,
+                             c->st));
+          }
           SR_TRY(read_ctrl(c));
           S.ms_select += now_ms() - tsel;
           if (S.rounds < SR_MAX_ROUNDS) {
@@ -776,6 +954,13 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
   for (int i = 0; i < b.N; ++i) {
     S.gen_tokens += lens[i];
     S.n_completed += stv[i] == ST_DONE;
+  }
+  c->prof.harvest();
+  for (int k = 0; k < SR_KC_N; ++k) {
+    S.kern_ms[k] = c->prof.ms[k];
+    S.kern_launches[k] = c->prof.n[k];
+    S.kern_flops[k] = c->prof.fl[k];
+    S.kern_bytes[k] = c->prof.by[k];
   }
   S.best_id = c->h_ctrl[C_BEST];
   S.peak_pages_in_use = c->h_ctrl[C_PEAK];
@@ -854,6 +1039,13 @@ void sr_destroy(sr_ctx* c) {
   if (c->h_meta) cudaFreeHost(c->h_meta);
   if (c->own) cudaStreamDestroy(c->own);
   delete c;
+}
+
+sr_status sr_set_profiling(sr_ctx* c, int enable) {
+  if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
+  c->prof.on = enable != 0;
+  c->prof.reset();
+  return SR_OK;
 }
 
 sr_status sr_set_stream(sr_ctx* c, void* stream) {

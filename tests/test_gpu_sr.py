@@ -13,6 +13,11 @@ from oracle.transformer import Decoder, Transformer
 
 pytestmark = pytest.mark.gpu
 LOGIT_TOL = 5e-2
+# Against the pure float32 oracle, rewards of a bf16-operand model can only be held to the deviation bf16
+# operand rounding itself causes: emulating exactly the kernels' rounding points inside the oracle moves
+# 2-layer Llama-width rewards by up to 2.8% of their rms (random init), so 6% of rms is the bound there; the
+# 1e-2 relative bound applies against the oracle computing with the same bf16 operands.
+BF16_REWARD_DEV = 6e-2
 
 
 @pytest.fixture(scope="module")
@@ -203,12 +208,14 @@ def _teacher_forced(sr, w, seed, prompt, n_steps):
                 if top[1] - top[0] > 2 * LOGIT_TOL:
                     assert q["tokens"][i][g] == int(np.argmax(z)), (i, g)
         rewards = sr.sr_score_partial(ctx, b, N)
-        ids = list(range(N))
-        rm = Transformer(w.rm, rw)
         from oracle.sr import score_sequences
-        want_r = score_sequences(rm, prompt, [q["tokens"][i][:q["lengths"][i]].tolist() for i in ids])
-        for a, bb in zip(rewards, want_r):
-            assert abs(a - bb) <= reward_tol(bb, want_r), (a, bb)
+        seqs = [q["tokens"][i][:q["lengths"][i]].tolist() for i in range(N)]
+        want_16 = score_sequences(Transformer(w.rm, rw, operand_rounding="bf16"), prompt, seqs)
+        for a, bb in zip(rewards, want_16):
+            assert abs(a - bb) <= reward_tol(bb, want_16), (a, bb)
+        want_32 = score_sequences(Transformer(w.rm, rw), prompt, seqs)
+        rms = float(np.sqrt(np.mean(want_32.astype(np.float64) ** 2)))
+        assert np.max(np.abs(rewards - want_32)) <= BF16_REWARD_DEV * rms
         sr.sr_batch_end(ctx, b)
     finally:
         sr.sr_destroy(ctx)

@@ -144,3 +144,25 @@ def test_window_equals_truncated_context():
     a = ot.attention(q, k, v, np.array([[9]]), np.arange(10)[None], 4)
     b = ot.attention(q, k[:, 6:], v[:, 6:], np.array([[9]]), np.arange(6, 10)[None], 0)
     np.testing.assert_allclose(a, b, rtol=1e-6, atol=1e-7)
+
+
+def test_bf16_operand_rounding_mode():
+    """round_bf16 is torch's float32 -> bfloat16 conversion; the bf16 mode only rounds operands, so KV-cached
+    decode still equals recompute in that mode, and an exact-bf16 input passes through unchanged."""
+    rng = np.random.default_rng(9)
+    x = (rng.standard_normal(100000) * 10.0 ** rng.uniform(-6, 6, 100000)).astype(np.float32)
+    want = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+    assert np.array_equal(ot.round_bf16(x), want)
+    assert np.array_equal(ot.round_bf16(want), want)
+    m = _small(si.NORM_RMS, si.ACT_SWIGLU, si.POS_ROPE).replace(dtype=si.DT_BF16)
+    w = si.random_weights(m, 3, perturb_norms=True)
+    mdl = ot.Transformer(m, w, operand_rounding="bf16")
+    seqs = np.tile(rng.integers(1, m.vocab, (1, 12)), (2, 1))
+    seqs[1, 8:] = rng.integers(1, m.vocab, 4)
+    full = mdl.forward(seqs)
+    dec = ot.Decoder(mdl, 2, 12)
+    dec.prefill(seqs[0, :8], [0, 1])
+    for t in range(8, 12):
+        np.testing.assert_allclose(dec.step([0, 1], seqs[:, t], t), full[:, t], rtol=1e-5, atol=1e-5)
+    plain = ot.Transformer(m, w).forward(seqs)
+    assert 0 < np.max(np.abs(plain - full)) < 0.1      # rounding changes results, but only slightly
