@@ -106,48 +106,56 @@ class ClockSampler:
 # ------------------------------------------------------------------------------------------------
 # CPU oracle sample (cpu_baseline and --impl reference)
 # ------------------------------------------------------------------------------------------------
-def oracle_sample(w: si.Workload, prompt_index: int = 0):
-    """Time the oracle's Algorithm 1 on a bounded sample of the workload: the same widths, vocabulary and
-    heads, 2 of the 32 layers, 4 candidates, a 64-token prompt prefix, 6 new tokens, one decision point at 3.
-    Its tokens/s is scaled to the full models by the ratio of matmul parameters touched per generated token
-    (generator + reward model), i.e. assuming cost linear in layers."""
-    from oracle.sr import SpeculativeRejection
-    from oracle.transformer import Transformer
-    L = 2
-    g = w.gen.replace(n_layers=L)
-    r = w.rm.replace(n_layers=L)
-    gw, rw = si.random_weights(g, 100, 0), si.random_weights(r, 100, 1)
-    gen, rm = Transformer(g, gw), Transformer(r, rw)
-    prompt = w.prompt(prompt_index)[:64]
-    N, max_new = 4, 6
-    t0 = time.perf_counter()
-    res = SpeculativeRejection(gen, rm, prompt, N, w.alpha, si.SCHED_FIXED, (3,), max_new, w.temperature,
-                               w.eos_bias, w.eos_id, 0).run()
-    dt = time.perf_counter() - t0
-    def per_tok(m):
-        layer = m.qkv_dim * m.d_model + m.d_model * m.n_heads * m.head_dim + \
-            (3 if m.gated else 2) * m.ffn_dim * m.d_model
-        return m.n_layers * layer + (m.vocab * m.d_model if m.has_lm_head else m.d_model)
-    scale = (per_tok(w.gen) + per_tok(w.rm)) / (per_tok(g) + per_tok(r))
-    tps = res.gen_tokens / dt / scale
-    try:
-        import threadpoolctl
-        cores = sum(p.get("num_threads", 0) for p in threadpoolctl.threadpool_info() if p.get("user_api") == "blas")
-    except Exception:
-        cores = os.cpu_count()
-    return {"value": tps, "unit": UNIT, "cores": cores or os.cpu_count(), "kind": "oracle",
-            "sample": (f"oracle Algorithm 1 on {w.name} widths with 2/32 layers, N=4, P=64, 6 new tokens, one "
-                       f"round at 3: {res.gen_tokens} tokens in {dt:.1f} s on the host, scaled by x{scale:.1f} "
-                       f"(matmul parameters per token, full / sample)")}
+class OracleSample:
+    """The oracle's Algorithm 1 on a bounded sample of the workload: the same widths, vocabulary and heads, 1 of
+    the 32 layers, 2 candidates, a 64-token prompt prefix, 4 new tokens, one decision point at 2.  Its tokens/s
+    is scaled to the full models by the ratio of matmul parameters touched per generated token (generator +
+    reward model), i.e. assuming cost linear in layers.  Models are built once; each run is timed."""
+    L, N, MAX_NEW, P = 1, 2, 4, 64
+
+    def __init__(self, w: si.Workload):
+        from oracle.transformer import Transformer
+        self.w = w
+        self.g = w.gen.replace(n_layers=self.L)
+        self.r = w.rm.replace(n_layers=self.L)
+        self.gen = Transformer(self.g, si.random_weights(self.g, 100, 0))
+        self.rm = Transformer(self.r, si.random_weights(self.r, 100, 1))
+
+        def per_tok(m):
+            layer = m.qkv_dim * m.d_model + m.d_model * m.n_heads * m.head_dim + \
+                (3 if m.gated else 2) * m.ffn_dim * m.d_model
+            return m.n_layers * layer + (m.vocab * m.d_model if m.has_lm_head else m.d_model)
+        self.scale = (per_tok(w.gen) + per_tok(w.rm)) / (per_tok(self.g) + per_tok(self.r))
+        try:
+            import threadpoolctl
+            self.cores = sum(p.get("num_threads", 0) for p in threadpoolctl.threadpool_info()
+                             if p.get("user_api") == "blas") or os.cpu_count()
+        except Exception:
+            self.cores = os.cpu_count()
+
+    def run(self, prompt_index: int = 0):
+        from oracle.sr import SpeculativeRejection
+        w = self.w
+        prompt = w.prompt(prompt_index)[:self.P]
+        t0 = time.perf_counter()
+        res = SpeculativeRejection(self.gen, self.rm, prompt, self.N, w.alpha, si.SCHED_FIXED, (2,), self.MAX_NEW,
+                                   w.temperature, w.eos_bias, w.eos_id, 0).run()
+        dt = time.perf_counter() - t0
+        return {"value": res.gen_tokens / dt / self.scale, "unit": UNIT, "cores": self.cores, "kind": "oracle",
+                "sample": (f"oracle Algorithm 1 on {w.name} widths with {self.L}/{w.gen.n_layers} layers, "
+                           f"N={self.N}, P={len(prompt)}, {self.MAX_NEW} new tokens, one round at 2: "
+                           f"{res.gen_tokens} tokens in {dt:.1f} s on the host, scaled by 1/{self.scale:.1f} "
+                           f"(matmul parameters per token, full / sample)")}
 
 
 def run_reference(args, w):
     rank, world, _ = dist_env()
     if rank != 0:
         return
+    smp = OracleSample(w)
     steps = []
     for k in range(args.warmup + args.steps):
-        s = oracle_sample(w, k % max(1, w.n_prompts))
+        s = smp.run(k % max(1, w.n_prompts))
         if k >= args.warmup:
             steps.append(s)
     v = statistics.mean(s["value"] for s in steps)
@@ -323,7 +331,7 @@ def main():
         "clocks": clocks, "e2e": e2e,
     }
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = oracle_sample(w)
+        line["cpu_baseline"] = OracleSample(w).run(0)
     print(json.dumps(line), flush=True)
 
 

@@ -45,7 +45,7 @@ typedef enum {
 enum { SR_NORM_RMS = 0, SR_NORM_LAYER = 1 };
 enum { SR_ACT_SWIGLU = 0, SR_ACT_GELU = 1, SR_ACT_GEGLU = 2 };
 enum { SR_POS_ROPE = 0, SR_POS_LEARNED = 1 };
-enum { SR_DT_F32 = 0, SR_DT_BF16 = 1 };
+enum { SR_DT_F32 = 0, SR_DT_BF16 = 1, SR_DT_F16 = 2 };
 enum { SR_SCHED_FIXED = 0, SR_SCHED_POOL_FULL = 1 };
 
 /*
@@ -70,7 +70,9 @@ typedef struct {
   int pos;  /* SR_POS_* */
   float rope_theta, norm_eps;
   int has_lm_head, has_scalar_head;
-  int dtype; /* SR_DT_*: weight, activation-operand and KV-cache type; accumulation is fp32 */
+  int dtype; /* SR_DT_*: type of the weight blob.  SR_DT_F32 models compute in fp32 on the CUDA cores;
+                SR_DT_BF16 / SR_DT_F16 models run fp16 operands and KV cache on the tensor cores with
+                fp32 accumulation (bf16 weights of magnitude >= 2^-17 are exact in fp16). */
 } sr_model_desc;
 
 /*
@@ -239,13 +241,13 @@ sr_status sr_k_sample(const float* logits, long long ld, int b, int vocab, const
 sr_status sr_k_rcut(const float* rewards, int b, float alpha, int k_override, float* r_cut_out, uint8_t* mask_out,
                     void* stream);
 
-/* Dense layer C = A W^T (fp32 accumulate).  dtype SR_DT_BF16 runs the tcgen05
- * tensor-core kernel, SR_DT_F32 the fp32 SIMT kernel.  A [M][K] (lda = K),
+/* Dense layer C = A W^T (fp32 accumulate).  dtype SR_DT_F16 or SR_DT_BF16 runs the
+ * tcgen05 tensor-core kernel, SR_DT_F32 the fp32 SIMT kernel.  A [M][K] (lda = K),
  * W [N][K], both of `dtype`.  epilogue: 0 store fp32 C [M][N]; 1 add into fp32
  * C [M][N]; 2 store C as `dtype`; 3 SwiGLU / 4 GeGLU on column pairs
  * interleaved in blocks of 32 (W rows 64j..64j+31 gate block j, 64j+32..64j+63
  * up block j) storing `dtype` C [M][N/2]; 5 tanh-GELU storing `dtype` C [M][N]
- * (3-5 bf16 only).  Needs K % 8 == 0, N % 32 == 0 (N % 64 for 3, 4). */
+ * (3-5 16-bit only).  Needs K % 8 == 0, N % 32 == 0 (N % 64 for 3, 4). */
 sr_status sr_k_gemm(int dtype, const void* A, const void* W, void* C, int M, int N, int K, int epilogue,
                     void* stream);
 
@@ -262,10 +264,10 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
  * optional shared prefix.  Sequence j owns query/key rows seq_off[j] ..
  * seq_off[j+1]-1 of q [rows][n_heads][dh] and k, v [rows][n_kv][dh], at positions
  * pos0 + (row - seq_off[j]); every sequence also sees the n_pre prefix keys
- * k_pre, v_pre [n_pre][n_kv][dh] at positions 0..n_pre-1.  bf16 only. */
-sr_status sr_k_prefill_attention(const void* q, const void* k, const void* v, const void* k_pre, const void* v_pre,
-                                 int n_pre, const int32_t* seq_off, int n_seq, int pos0, int n_heads, int n_kv_heads,
-                                 int head_dim, int window, void* out, void* stream);
+ * k_pre, v_pre [n_pre][n_kv][dh] at positions 0..n_pre-1.  dtype SR_DT_F16 or SR_DT_BF16. */
+sr_status sr_k_prefill_attention(int dtype, const void* q, const void* k, const void* v, const void* k_pre,
+                                 const void* v_pre, int n_pre, const int32_t* seq_off, int n_seq, int pos0,
+                                 int n_heads, int n_kv_heads, int head_dim, int window, void* out, void* stream);
 
 #ifdef __cplusplus
 }

@@ -90,7 +90,7 @@ _SIG = {
     "sr_k_rcut": [_P, _I, _F, _I, _P, _P, _P],
     "sr_k_gemm": [_I, _P, _P, _P, _I, _I, _I, _I, _P],
     "sr_k_decode_attention": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P, _P],
-    "sr_k_prefill_attention": [_P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _P, _P],
+    "sr_k_prefill_attention": [_I, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _P, _P],
 }
 
 
@@ -273,8 +273,8 @@ def sr_k_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens,
                                      _stream(stream)))
 
 
-def sr_k_prefill_attention(q, k, v, k_pre, v_pre, n_pre, seq_off, n_seq, pos0, n_heads, n_kv_heads, head_dim, window,
-                           out, stream=None):
-    _check(LIB.sr_k_prefill_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(k_pre), _ptr(v_pre), n_pre, _ptr(seq_off),
+def sr_k_prefill_attention(dtype, q, k, v, k_pre, v_pre, n_pre, seq_off, n_seq, pos0, n_heads, n_kv_heads, head_dim,
+                           window, out, stream=None):
+    _check(LIB.sr_k_prefill_attention(dtype, _ptr(q), _ptr(k), _ptr(v), _ptr(k_pre), _ptr(v_pre), n_pre, _ptr(seq_off),
                                       n_seq, pos0, n_heads, n_kv_heads, head_dim, window, _ptr(out),
                                       _stream(stream)))

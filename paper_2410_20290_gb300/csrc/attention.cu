@@ -14,6 +14,9 @@
 // Prefill (k_prefill_attn): flash-attention style over packed variable-length sequences with a
 // shared prefix (the prompt's KV) -- 64 query rows x one head per CTA, 64-key blocks staged by
 // cp.async, bf16 mma.sync m16n8k16 with fp32 accumulation, online softmax in registers.
+#include <algorithm>
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace sr {
@@ -174,39 +177,247 @@ __device__ __forceinline__ void ldm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& 
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"(addr));
 }
+template <typename T>
 __device__ __forceinline__ void mma16816(float* c, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
                                          uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  if constexpr (std::is_same<T, bf16>::value)
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  else
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// (a, b) -> packed bf16 (hi) and the packed bf16 rounding of the remainders (lo)
-__device__ __forceinline__ void split_bf16(float a, float b, uint32_t& hi, uint32_t& lo) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-  const float2 hf = __bfloat1622float2(h);
-  const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
-  hi = *reinterpret_cast<const uint32_t*>(&h);
-  lo = *reinterpret_cast<const uint32_t*>(&l);
+// (a, b) -> packed 16-bit pair (hi) and the packed rounding of the remainders (lo)
+template <typename T>
+__device__ __forceinline__ void split16(float a, float b, uint32_t& hi, uint32_t& lo) {
+  if constexpr (std::is_same<T, bf16>::value) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    const float2 hf = __bfloat1622float2(h);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
+    hi = *reinterpret_cast<const uint32_t*>(&h);
+    lo = *reinterpret_cast<const uint32_t*>(&l);
+  } else {
+    const __half2 h = __floats2half2_rn(a, b);
+    const float2 hf = __half22float2(h);
+    const __half2 l = __floats2half2_rn(a - hf.x, b - hf.y);
+    hi = *reinterpret_cast<const uint32_t*>(&h);
+    lo = *reinterpret_cast<const uint32_t*>(&l);
+  }
+}
+template <typename T>
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  if constexpr (std::is_same<T, bf16>::value) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&h);
+  } else {
+    const __half2 h = __floats2half2_rn(fminf(fmaxf(a, -65504.f), 65504.f), fminf(fmaxf(b, -65504.f), 65504.f));
+    return *reinterpret_cast<const uint32_t*>(&h);
+  }
+}
+
+
+// Tensor-core paged decode attention for 16-bit KV (G <= 8 query heads per kv head).
+// One CTA per (kv head, slot, split); warp w takes pages w, w+4, ... of the split.  Each page's K and V
+// blocks (16 positions x dh, contiguous in the pool) are copied by a 2-deep per-warp cp.async pipeline
+// into padded shared memory; S^T = K Q^T is one m16n8 tile per page (16 positions x 8 head columns,
+// the G real heads plus zero padding), the online softmax runs per head column across the 8 lanes
+// holding its 16 positions, and O^T += V^T P^T adds dh/16 tiles with P carried as an fp16/bf16
+// hi + lo pair.  Warps merge their (m, l, O) through shared memory at the end.
+template <typename T, int DH, int G>
+__global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q, const T* __restrict__ pool,
+                                                        const int* __restrict__ pt, int pt_stride,
+                                                        const int* __restrict__ slot_ids,
+                                                        const int* __restrict__ lens, int Hkv, float scale_log2,
+                                                        int window, int max_splits, T* __restrict__ out,
+                                                        float* __restrict__ part) {
+  static_assert(G >= 1 && G <= 8 && DH % 16 == 0, "shape");
+  constexpr int LDS = DH + 8;                  // padded smem row (elements): conflict-free ldmatrix
+  constexpr int BLK = PAGE * LDS;              // one K or V page block in smem
+  constexpr int WARP_ELEMS = 2 * 2 * BLK + 2 * 8 * PAGE;  // 2 stages x (K, V) + P hi / lo [8][16]
+  constexpr int KS = DH / 16;
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  T* sw = reinterpret_cast<T*>(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
+  T* wbase = sw + warp * WARP_ELEMS;
+  uint16_t* sPh = reinterpret_cast<uint16_t*>(wbase + 4 * BLK);
+  uint16_t* sPl = sPh + 8 * PAGE;
+
+  const int h = blockIdx.x, s = blockIdx.y, split = blockIdx.z;
+  const int Hq = Hkv * G;
+  const int L = lens[s];
+  const int t_lo = window > 0 ? max(0, L - window) : 0;
+  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  if (split >= nsplit) return;
+  const int t_begin = t_lo + split * SPLIT, t_end = min(L, t_begin + SPLIT);
+  const int p_first = t_begin / PAGE, n_pages = (t_end - 1) / PAGE - p_first + 1;
+  const int my_pages = n_pages > warp ? (n_pages - warp + 3) / 4 : 0;
+  const int* ptrow = pt + (size_t)slot_ids[s] * pt_stride;
+  const size_t page_elems = (size_t)2 * Hkv * PAGE * DH;
+  const size_t v_off = (size_t)Hkv * PAGE * DH;
+
+  // B fragments of Q^T (k = dim, n = head): lane holds head g (zero when g >= G)
+  uint32_t qb[KS][2];
+  {
+    const T* qh = q + ((size_t)s * Hq + h * G + (g < G ? g : 0)) * DH;
+#pragma unroll
+    for (int k = 0; k < KS; ++k) {
+      qb[k][0] = g < G ? *reinterpret_cast<const uint32_t*>(qh + k * 16 + 2 * t4) : 0u;
+      qb[k][1] = g < G ? *reinterpret_cast<const uint32_t*>(qh + k * 16 + 8 + 2 * t4) : 0u;
+    }
+  }
+  auto issue = [&](int i, int stage) {
+    const int page = ptrow[p_first + warp + 4 * i];
+    const T* srcK = pool + (size_t)page * page_elems + (size_t)h * PAGE * DH;
+    const T* srcV = srcK + v_off;
+    T* dK = wbase + stage * 2 * BLK;
+    T* dV = dK + BLK;
+#pragma unroll
+    for (int c = lane; c < PAGE * DH / 8; c += 32) {
+      const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+      cp_async16(dK + row * LDS + col, srcK + row * DH + col, true);
+      cp_async16(dV + row * LDS + col, srcV + row * DH + col, true);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+
+  float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};
+  float o[KS][4];
+#pragma unroll
+  for (int i = 0; i < KS; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+
+  if (my_pages > 0) issue(0, 0);
+  if (my_pages > 1) issue(1, 1);
+  for (int i = 0; i < my_pages; ++i) {
+    const int stage = i & 1;
+    if (i + 1 < my_pages) asm volatile("cp.async.wait_group 1;" ::: "memory");
+    else asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncwarp();
+    const T* sK = wbase + stage * 2 * BLK;
+    const T* sV = sK + BLK;
+    // S^T = K Q^T : 16 positions x 8 head columns
+    float sc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int k = 0; k < KS; ++k) {
+      uint32_t a0, a1, a2, a3;
+      ldm_x4(smem_addr(sK + (lane & 15) * LDS + k * 16 + (lane >> 4) * 8), a0, a1, a2, a3);
+      mma16816<T>(sc, a0, a1, a2, a3, qb[k][0], qb[k][1]);
+    }
+    const int tok0 = (p_first + warp + 4 * i) * PAGE + g;
+    const bool v0 = tok0 >= t_begin && tok0 < t_end, v1 = tok0 + 8 >= t_begin && tok0 + 8 < t_end;
+    float corr[2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {      // head columns 2 t4 + j
+      const float x0 = v0 ? sc[j] * scale_log2 : -INFINITY;
+      const float x1 = v1 ? sc[2 + j] * scale_log2 : -INFINITY;
+      float bm = fmaxf(x0, x1);
+      bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 4));
+      bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 8));
+      bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 16));
+      const float mn = fmaxf(m[j], bm);
+      const float base = (mn == -INFINITY) ? 0.f : mn;
+      corr[j] = exp2f(m[j] - base);
+      const float p0 = exp2f(x0 - base), p1 = exp2f(x1 - base);
+      float ps = p0 + p1;
+      ps += __shfl_xor_sync(0xffffffffu, ps, 4);
+      ps += __shfl_xor_sync(0xffffffffu, ps, 8);
+      ps += __shfl_xor_sync(0xffffffffu, ps, 16);
+      l[j] = l[j] * corr[j] + ps;
+      m[j] = mn;
+      // P[head][position] as hi + lo 16-bit values
+      const int hc = 2 * t4 + j;
+      uint32_t hi, lo;
+      split16<T>(p0, p1, hi, lo);
+      sPh[hc * PAGE + g] = (uint16_t)(hi & 0xFFFFu);
+      sPh[hc * PAGE + g + 8] = (uint16_t)(hi >> 16);
+      sPl[hc * PAGE + g] = (uint16_t)(lo & 0xFFFFu);
+      sPl[hc * PAGE + g + 8] = (uint16_t)(lo >> 16);
+    }
+#pragma unroll
+    for (int mt = 0; mt < KS; ++mt) {
+      o[mt][0] *= corr[0], o[mt][1] *= corr[1];
+      o[mt][2] *= corr[0], o[mt][3] *= corr[1];
+    }
+    __syncwarp();
+    // B fragments of P^T (k = position, n = head g)
+    const uint32_t bh0 = *reinterpret_cast<const uint32_t*>(sPh + g * PAGE + 2 * t4);
+    const uint32_t bh1 = *reinterpret_cast<const uint32_t*>(sPh + g * PAGE + 8 + 2 * t4);
+    const uint32_t bl0 = *reinterpret_cast<const uint32_t*>(sPl + g * PAGE + 2 * t4);
+    const uint32_t bl1 = *reinterpret_cast<const uint32_t*>(sPl + g * PAGE + 8 + 2 * t4);
+    // O^T += V^T P^T : dims in m16 tiles
+#pragma unroll
+    for (int mt = 0; mt < KS; ++mt) {
+      uint32_t a0, a1, a2, a3;
+      const int mi = lane >> 3, r = lane & 7;
+      ldm_x4_t(smem_addr(sV + (r + ((mi >> 1) << 3)) * LDS + mt * 16 + (mi & 1) * 8), a0, a1, a2, a3);
+      mma16816<T>(o[mt], a0, a1, a2, a3, bh0, bh1);
+      mma16816<T>(o[mt], a0, a1, a2, a3, bl0, bl1);
+    }
+    __syncwarp();
+    if (i + 2 < my_pages) issue(i + 2, stage);
+  }
+  // merge the 4 warps' partial softmax states
+  __syncthreads();
+  float* sm = reinterpret_cast<float*>(smem_raw);            // [4][8] maxima
+  float* sl = sm + 32;                                       // [4][8] sums
+  float* so = sl + 32;                                       // [4][DH][8] O^T
+  if (g == 0) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) sm[warp * 8 + 2 * t4 + j] = m[j], sl[warp * 8 + 2 * t4 + j] = l[j];
+  }
+#pragma unroll
+  for (int mt = 0; mt < KS; ++mt) {
+    float* ow = so + (size_t)warp * DH * 8;
+    ow[(mt * 16 + g) * 8 + 2 * t4] = o[mt][0];
+    ow[(mt * 16 + g) * 8 + 2 * t4 + 1] = o[mt][1];
+    ow[(mt * 16 + g + 8) * 8 + 2 * t4] = o[mt][2];
+    ow[(mt * 16 + g + 8) * 8 + 2 * t4 + 1] = o[mt][3];
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < G * DH; idx += 128) {
+    const int j = idx / DH, d = idx % DH;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, sm[w * 8 + j]);
+    float Lsum = 0.f, O = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float wt = (sm[w * 8 + j] == -INFINITY) ? 0.f : exp2f(sm[w * 8 + j] - M);
+      Lsum += sl[w * 8 + j] * wt;
+      O += so[((size_t)w * DH + d) * 8 + j] * wt;
+    }
+    const int hq = h * G + j;
+    if (nsplit == 1) {
+      out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
+    } else {
+      float* pp = part + (((size_t)s * Hq + hq) * max_splits + split) * (DH + 2);
+      pp[d] = O;
+      if (d == 0) pp[DH] = M, pp[DH + 1] = Lsum;
+    }
+  }
 }
 
 constexpr int BQ = 64, BKV = 64;
 
-template <int DH, int DV>
-__global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q, const bf16* __restrict__ k,
-                                                      const bf16* __restrict__ v, const bf16* __restrict__ kpre,
-                                                      const bf16* __restrict__ vpre, int npre,
+template <typename T, int DH, int DV>
+__global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, const T* __restrict__ k,
+                                                      const T* __restrict__ v, const T* __restrict__ kpre,
+                                                      const T* __restrict__ vpre, int npre,
                                                       const int* __restrict__ seq_off,
                                                       const int* __restrict__ tile_seq,
                                                       const int* __restrict__ tile_q0, int pos0, int Hq, int Hkv,
-                                                      float scale_log2, int window, bf16* __restrict__ out) {
+                                                      float scale_log2, int window, T* __restrict__ out) {
   constexpr int LD = DH + 8, LDV = DV + 8;
   extern __shared__ __align__(16) uint8_t smem_raw[];
-  bf16* sQ = reinterpret_cast<bf16*>(smem_raw);
-  bf16* sK = sQ + BQ * LD;
-  bf16* sV = sK + BKV * LD;
+  T* sQ = reinterpret_cast<T*>(smem_raw);
+  T* sK = sQ + BQ * LD;
+  T* sV = sK + BKV * LD;
 
   const int tile = blockIdx.x, hq = blockIdx.y, dvo = blockIdx.z * DV;
   const int j = tile_seq[tile], q0 = tile_q0[tile];
@@ -219,7 +430,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q
   for (int c = tid; c < BQ * (DH / 8); c += 128) {
     const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
     const bool ok = q0 + row < nrows;
-    const bf16* src = ok ? q + (size_t)(r0 + q0 + row) * qstride + (size_t)hq * DH + col : q;
+    const T* src = ok ? q + (size_t)(r0 + q0 + row) * qstride + (size_t)hq * DH + col : q;
     cp_async16(sQ + row * LD + col, src, ok);
   }
 
@@ -244,18 +455,18 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q
     if (window > 0 && kpos0 + kcount - 1 <= qpos_min - window) continue;  // whole block left of every window
     if (kpos0 > qpos_max) continue;
     __syncthreads();  // previous block's smem reads are done
-    const bf16* ksrc = is_pre ? kpre : k + (size_t)r0 * kstride;
-    const bf16* vsrc = is_pre ? vpre : v + (size_t)r0 * kstride;
+    const T* ksrc = is_pre ? kpre : k + (size_t)r0 * kstride;
+    const T* vsrc = is_pre ? vpre : v + (size_t)r0 * kstride;
     for (int c = tid; c < BKV * (DH / 8); c += 128) {
       const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
       const bool ok = row < kcount;
-      const bf16* src = ok ? ksrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + col : ksrc;
+      const T* src = ok ? ksrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + col : ksrc;
       cp_async16(sK + row * LD + col, src, ok);
     }
     for (int c = tid; c < BKV * (DV / 8); c += 128) {
       const int row = c / (DV / 8), col = (c % (DV / 8)) * 8;
       const bool ok = row < kcount;
-      const bf16* src = ok ? vsrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + dvo + col : vsrc;
+      const T* src = ok ? vsrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + dvo + col : vsrc;
       cp_async16(sV + row * LDV + col, src, ok);
     }
     cp_async_wait_all();
@@ -274,8 +485,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q
         uint32_t b0, b1, b2, b3;
         ldm_x4(smem_addr(sK + (np * 16 + (lane & 7) + ((lane >> 4) << 3)) * LD + kk * 16 + ((lane >> 3) & 1) * 8), b0,
                b1, b2, b3);
-        mma16816(sc[2 * np], a0, a1, a2, a3, b0, b1);
-        mma16816(sc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+        mma16816<T>(sc[2 * np], a0, a1, a2, a3, b0, b1);
+        mma16816<T>(sc[2 * np + 1], a0, a1, a2, a3, b2, b3);
       }
     }
     // mask, scale, online softmax
@@ -326,19 +537,19 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q
 #pragma unroll
     for (int kk = 0; kk < BKV / 16; ++kk) {
       uint32_t ah[4], al[4];
-      split_bf16(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
-      split_bf16(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
-      split_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
-      split_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
+      split16<T>(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+      split16<T>(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+      split16<T>(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+      split16<T>(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
 #pragma unroll
       for (int dp = 0; dp < DV / 16; ++dp) {
         uint32_t b0, b1, b2, b3;
         ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LDV + dp * 16 + (lane >> 4) * 8), b0,
                  b1, b2, b3);
-        mma16816(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
-        mma16816(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
-        mma16816(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
-        mma16816(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
+        mma16816<T>(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
+        mma16816<T>(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+        mma16816<T>(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
+        mma16816<T>(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
       }
     }
   }
@@ -353,12 +564,10 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const bf16* __restrict__ q
     const int qi = qi_a + 8 * r;
     if (qi >= nrows) continue;
     const float inv = lrow[r] > 0.f ? 1.f / lrow[r] : 0.f;
-    bf16* dst = out + (size_t)(r0 + qi) * qstride + (size_t)hq * DH + dvo;
+    T* dst = out + (size_t)(r0 + qi) * qstride + (size_t)hq * DH + dvo;
 #pragma unroll
-    for (int nt = 0; nt < DV / 8; ++nt) {
-      const __nv_bfloat162 h = __floats2bfloat162_rn(o[nt][2 * r] * inv, o[nt][2 * r + 1] * inv);
-      *reinterpret_cast<__nv_bfloat162*>(dst + nt * 8 + 2 * t4) = h;
-    }
+    for (int nt = 0; nt < DV / 8; ++nt)
+      *reinterpret_cast<uint32_t*>(dst + nt * 8 + 2 * t4) = pack2<T>(o[nt][2 * r] * inv, o[nt][2 * r + 1] * inv);
   }
 }
 
@@ -414,6 +623,30 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
 }
 
 template <typename T, int DH, int G>
+sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
+                           const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
+                           cudaStream_t st) {
+  constexpr int LDS = DH + 8;
+  const size_t smem = std::max<size_t>((size_t)4 * (2 * 2 * PAGE * LDS + 2 * 8 * PAGE) * sizeof(T),
+                                       (size_t)(64 + 4 * DH * 8) * sizeof(float));
+  static bool attr_set = false;
+  if (!attr_set) {
+    SR_CUDA(cudaFuncSetAttribute(k_decode_attn_tc<T, DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    attr_set = true;
+  }
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
+  dim3 grid(Hkv, b, max_splits);
+  k_decode_attn_tc<T, DH, G><<<grid, 128, smem, st>>>((const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
+                                                       scale_log2, window, max_splits, (T*)out, part);
+  SR_LAUNCH();
+  if (max_splits > 1) {
+    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, (T*)out);
+    SR_LAUNCH();
+  }
+  return SR_OK;
+}
+
+template <typename T, int DH, int G>
 sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
                         const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
                         cudaStream_t st) {
@@ -429,20 +662,21 @@ sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_s
   return SR_OK;
 }
 
-template <int DH, int DV>
-sr_status prefill_t(const bf16* q, const bf16* k, const bf16* v, const bf16* kpre, const bf16* vpre, int npre,
+template <typename T, int DH, int DV>
+sr_status prefill_t(const void* q, const void* k, const void* v, const void* kpre, const void* vpre, int npre,
                     const int* seq_off, const int* tile_seq, const int* tile_q0, int n_tiles, int pos0, int Hq,
-                    int Hkv, int window, bf16* out, cudaStream_t st) {
-  const size_t smem = (size_t)(BQ * (DH + 8) + BKV * (DH + 8) + BKV * (DV + 8)) * sizeof(bf16);
+                    int Hkv, int window, void* out, cudaStream_t st) {
+  const size_t smem = (size_t)(BQ * (DH + 8) + BKV * (DH + 8) + BKV * (DV + 8)) * sizeof(T);
   static bool attr_set = false;
   if (!attr_set) {
-    SR_CUDA(cudaFuncSetAttribute(k_prefill_attn<DH, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    SR_CUDA(cudaFuncSetAttribute(k_prefill_attn<T, DH, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid(n_tiles, Hq, DH / DV);
-  k_prefill_attn<DH, DV><<<grid, 128, smem, st>>>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, pos0, Hq,
-                                                   Hkv, scale_log2, window, out);
+  k_prefill_attn<T, DH, DV><<<grid, 128, smem, st>>>((const T*)q, (const T*)k, (const T*)v, (const T*)kpre,
+                                                      (const T*)vpre, npre, seq_off, tile_seq, tile_q0, pos0, Hq, Hkv,
+                                                      scale_log2, window, (T*)out);
   SR_LAUNCH();
   return SR_OK;
 }
@@ -454,26 +688,33 @@ size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits) {
   return (size_t)b * Hq * max_splits * (dh + 2);
 }
 
-sr_status launch_decode_attention(int dtype, const void* q, const void* pool_layer, const int* pt, int pt_stride,
+sr_status launch_decode_attention(int et, const void* q, const void* pool_layer, const int* pt, int pt_stride,
                                   const int* ids, const int* lens, int b, int Hq, int Hkv, int dh, int window,
                                   void* out, float* part, int max_splits, cudaStream_t st) {
   if (b == 0) return SR_OK;
   const int G = Hq / Hkv;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "decode attention: n_heads %% n_kv_heads != 0");
   if (max_splits > 1 && !part) return set_err(SR_ERR_INVALID_ARG, "decode attention: split partial buffer missing");
-#define SR_DEC(T, D, GG)                                                                                      \
-  if (dh == D && G == GG)                                                                                     \
+#define SR_DEC(T, D, GG)                                                                                          \
+  if (dh == D && G == GG)                                                                                         \
     return decode_attn_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
                                    st);
-  if (dtype == SR_DT_BF16) {
-    SR_DEC(bf16, 128, 4) SR_DEC(bf16, 128, 1) SR_DEC(bf16, 128, 2) SR_DEC(bf16, 128, 8)
-    SR_DEC(bf16, 64, 1) SR_DEC(bf16, 64, 4) SR_DEC(bf16, 32, 1)
+#define SR_DECT(T, D, GG)                                                                                          \
+  if (dh == D && G == GG)                                                                                            \
+    return decode_attn_tc_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
+                                      st);
+  if (et == SR_DT_F16) {
+    SR_DECT(f16, 128, 4) SR_DECT(f16, 128, 1) SR_DECT(f16, 128, 2) SR_DECT(f16, 128, 8)
+    SR_DECT(f16, 64, 1) SR_DECT(f16, 64, 4) SR_DECT(f16, 32, 1)
+  } else if (et == SR_DT_BF16) {
+    SR_DECT(bf16, 128, 4) SR_DECT(bf16, 128, 1) SR_DECT(bf16, 64, 1)
   } else {
     SR_DEC(float, 32, 1) SR_DEC(float, 32, 2) SR_DEC(float, 32, 4) SR_DEC(float, 64, 1) SR_DEC(float, 128, 1)
     SR_DEC(float, 8, 1) SR_DEC(float, 8, 2) SR_DEC(float, 8, 4)
   }
 #undef SR_DEC
-  return set_err(SR_ERR_UNSUPPORTED, "decode attention: head_dim %d with group %d (dtype %d) not built", dh, G, dtype);
+#undef SR_DECT
+  return set_err(SR_ERR_UNSUPPORTED, "decode attention: head_dim %d with group %d (type %d) not built", dh, G, et);
 }
 
 sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* kpre,
@@ -494,19 +735,31 @@ sr_status launch_prefill_attention_f32(const float* q, const float* k, const flo
   return SR_OK;
 }
 
-sr_status launch_prefill_attention(const bf16* q, const bf16* k, const bf16* v, const bf16* kpre, const bf16* vpre,
-                                   int npre, const int* seq_off, int n_seq, const int* tile_seq, const int* tile_q0,
-                                   int n_tiles, int pos0, int Hq, int Hkv, int dh, int window, bf16* out,
-                                   cudaStream_t st) {
+sr_status launch_prefill_attention(int et, const void* q, const void* k, const void* v, const void* kpre,
+                                   const void* vpre, int npre, const int* seq_off, int n_seq, const int* tile_seq,
+                                   const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
+                                   void* out, cudaStream_t st) {
   (void)n_seq;
   if (n_tiles == 0) return SR_OK;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "prefill attention: n_heads %% n_kv_heads != 0");
-  switch (dh) {
-    case 32: return prefill_t<32, 32>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
-    case 64: return prefill_t<64, 64>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
-    case 128: return prefill_t<128, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
-    case 256: return prefill_t<256, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, window, out, st);
+  if (et != SR_DT_F16 && et != SR_DT_BF16) return set_err(SR_ERR_INVALID_ARG, "prefill attention: 16-bit types only");
+#define SR_PRE(T)                                                                                                      \
+  switch (dh) {                                                                                                        \
+    case 32: return prefill_t<T, 32, 32>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, \
+                                         window, out, st);                                                            \
+    case 64: return prefill_t<T, 64, 64>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, \
+                                         window, out, st);                                                            \
+    case 128: return prefill_t<T, 128, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, \
+                                            Hkv, window, out, st);                                                    \
+    case 256: return prefill_t<T, 256, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, \
+                                            Hkv, window, out, st);                                                    \
   }
+  if (et == SR_DT_F16) {
+    SR_PRE(f16)
+  } else {
+    SR_PRE(bf16)
+  }
+#undef SR_PRE
   return set_err(SR_ERR_UNSUPPORTED, "prefill attention: head_dim %d not built", dh);
 }
 

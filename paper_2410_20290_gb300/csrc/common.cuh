@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -10,6 +11,11 @@
 namespace sr {
 
 typedef __nv_bfloat16 bf16;
+typedef __half f16;
+// Element types of device tensors use the SR_DT_* codes: SR_DT_F32, SR_DT_BF16, SR_DT_F16.  Models
+// whose weights arrive in bf16 (or fp16) run with fp16 operands and KV cache: every bf16 value of
+// magnitude >= 2^-17 is exact in fp16, and fp16's 11-bit significand makes the rounding of
+// activations fed to the tensor cores 8x finer than bf16's, at the same tensor-core rate.
 constexpr int PAGE = 16;            // positions per KV page
 constexpr int MAX_BATCH = 4096;     // largest N handled by the single-CTA control kernels
 
@@ -37,12 +43,16 @@ sr_status set_err(sr_status s, const char* fmt, ...);
 // ---------------------------------------------------------------------------------------------
 __device__ __forceinline__ float to_f(float x) { return x; }
 __device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ float to_f(f16 x) { return __half2float(x); }
 template <typename T>
 __device__ __forceinline__ T f_to(float x);
 template <>
 __device__ __forceinline__ float f_to<float>(float x) { return x; }
 template <>
 __device__ __forceinline__ bf16 f_to<bf16>(float x) { return __float2bfloat16_rn(x); }
+// fp16 conversions saturate at the largest finite value instead of overflowing to infinity
+template <>
+__device__ __forceinline__ f16 f_to<f16>(float x) { return __float2half_rn(fminf(fmaxf(x, -65504.f), 65504.f)); }
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -107,13 +117,22 @@ __device__ __forceinline__ float key_float(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
 
+// Run `body` with T bound to the device element type of code `et` (SR_DT_*).
+#define SR_DISPATCH_ET(et, T, body)                                                       \
+  switch (et) {                                                                           \
+    case SR_DT_F32: { typedef float T; body; } break;                                     \
+    case SR_DT_BF16: { typedef ::sr::bf16 T; body; } break;                               \
+    case SR_DT_F16: { typedef ::sr::f16 T; body; } break;                                 \
+    default: return ::sr::set_err(SR_ERR_INVALID_ARG, "unknown element type %d", (int)(et)); \
+  }
+
 // ---------------------------------------------------------------------------------------------
 // host launchers implemented in the kernel files
 // ---------------------------------------------------------------------------------------------
 enum Epi { EPI_F32 = 0, EPI_ADD_F32 = 1, EPI_STORE = 2, EPI_SWIGLU = 3, EPI_GEGLU = 4, EPI_GELU = 5 };
 
-// gemm_tc.cu: bf16 tcgen05 GEMM, C = A W^T; needs sm_100+ tensor memory.
-sr_status gemm_bf16(const bf16* A, const bf16* W, void* C, int M, int N, int K, int epi, cudaStream_t st);
+// gemm_tc.cu: tcgen05 GEMM, C = A W^T, A and W both bf16 or both fp16 (et = SR_DT_BF16 / SR_DT_F16).
+sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, int K, int epi, cudaStream_t st);
 // gemm_f32.cu: fp32 SIMT GEMM (epilogues EPI_F32, EPI_ADD_F32, EPI_STORE).
 sr_status gemm_f32(const float* A, const float* W, float* C, int M, int N, int K, int epi, cudaStream_t st);
 
@@ -151,10 +170,12 @@ size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits);
 sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* k_pre,
                                        const float* v_pre, int n_pre, const int* seq_off, int n_seq, int rows,
                                        int pos0, int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st);
-sr_status launch_prefill_attention(const bf16* q, const bf16* k, const bf16* v, const bf16* k_pre,
-                                   const bf16* v_pre, int n_pre, const int* seq_off, int n_seq, const int* tile_seq,
+sr_status launch_prefill_attention(int et, const void* q, const void* k, const void* v, const void* k_pre,
+                                   const void* v_pre, int n_pre, const int* seq_off, int n_seq, const int* tile_seq,
                                    const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
-                                   bf16* out, cudaStream_t st);
+                                   void* out, cudaStream_t st);
+// elementwise.cu: in-place bf16 -> fp16 conversion of n elements (weights at load)
+sr_status launch_bf16_to_f16(void* p, size_t n, cudaStream_t st);
 
 // select.cu -- device control words and candidate states
 enum Ctrl { C_NLIVE = 0, C_TOP, C_NRSET, C_ERR, C_PEAK, C_K, C_KRAISED, C_NACC, C_BEST, C_NPOOL, C_N };

@@ -4,6 +4,8 @@
 //
 // These compute the per-position parts of the generator and reward model of Section 3; the KV
 // append is the paged cache of the Section 5 engine ("pre-allocates the corresponding KV cache").
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace sr {
@@ -177,30 +179,34 @@ __global__ void k_copy_page(T* pool, long long layer_stride, int page_elems, int
   for (int i = threadIdx.x; i < page_elems; i += blockDim.x) t[i] = s[i];
 }
 
+// bf16 bit patterns -> fp16 bit patterns, in place (exact for |x| in [2^-17, 65504]; smaller
+// magnitudes round to the fp16 subnormal grid, larger ones saturate)
+__global__ void k_bf16_to_f16(uint16_t* p, size_t n) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    const float v = __uint_as_float((uint32_t)p[i] << 16);
+    const f16 h = f_to<f16>(v);
+    p[i] = *reinterpret_cast<const uint16_t*>(&h);
+  }
+}
+
 int threads_for(int d) { return d >= 1024 ? 256 : (d >= 256 ? 128 : 64); }
 
 }  // namespace
 
-sr_status launch_embed(int dtype, const void* tok_emb, const void* pos_emb, const int* tokens, const int* positions,
+sr_status launch_embed(int et, const void* tok_emb, const void* pos_emb, const int* tokens, const int* positions,
                        int M, int d, float* x, cudaStream_t st) {
   if (M == 0) return SR_OK;
-  if (dtype == SR_DT_BF16)
-    k_embed<bf16><<<M, threads_for(d), 0, st>>>((const bf16*)tok_emb, (const bf16*)pos_emb, tokens, positions, d, x);
-  else
-    k_embed<float><<<M, threads_for(d), 0, st>>>((const float*)tok_emb, (const float*)pos_emb, tokens, positions, d,
-                                                 x);
+  SR_DISPATCH_ET(et, T, (k_embed<T><<<M, threads_for(d), 0, st>>>((const T*)tok_emb, (const T*)pos_emb, tokens,
+                                                                  positions, d, x)));
   SR_LAUNCH();
   return SR_OK;
 }
 
-sr_status launch_norm(int dtype, int norm, const float* x, const void* w, const void* b, float eps, int M, int d,
+sr_status launch_norm(int et, int norm, const float* x, const void* w, const void* b, float eps, int M, int d,
                       void* out, cudaStream_t st) {
   if (M == 0) return SR_OK;
   const int ln = norm == SR_NORM_LAYER;
-  if (dtype == SR_DT_BF16)
-    k_norm<bf16><<<M, threads_for(d), 0, st>>>(x, (const bf16*)w, (const bf16*)b, eps, d, ln, (bf16*)out);
-  else
-    k_norm<float><<<M, threads_for(d), 0, st>>>(x, (const float*)w, (const float*)b, eps, d, ln, (float*)out);
+  SR_DISPATCH_ET(et, T, (k_norm<T><<<M, threads_for(d), 0, st>>>(x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
   SR_LAUNCH();
   return SR_OK;
 }
@@ -212,51 +218,45 @@ sr_status launch_rope_table(float2* tab, int max_pos, int head_dim, double theta
   return SR_OK;
 }
 
-sr_status launch_rope_store(int dtype, const float* qkv, int M, const int* positions, const float2* rope, int Hq,
+sr_status launch_rope_store(int et, const float* qkv, int M, const int* positions, const float2* rope, int Hq,
                             int Hkv, int dh, void* q_out, void* k_out, void* v_out, KvSink sink, cudaStream_t st) {
   if (M == 0) return SR_OK;
-  if (dtype == SR_DT_BF16)
-    k_rope_store<bf16><<<M, 128, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (bf16*)q_out, (bf16*)k_out,
-                                          (bf16*)v_out, sink);
-  else
-    k_rope_store<float><<<M, 128, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (float*)q_out, (float*)k_out,
-                                           (float*)v_out, sink);
+  SR_DISPATCH_ET(et, T, (k_rope_store<T><<<M, 128, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (T*)q_out, (T*)k_out,
+                                                            (T*)v_out, sink)));
   SR_LAUNCH();
   return SR_OK;
 }
 
-sr_status launch_act(int dtype, int act, const float* in, int M, int F, void* out, cudaStream_t st) {
+sr_status launch_act(int et, int act, const float* in, int M, int F, void* out, cudaStream_t st) {
   if (M == 0) return SR_OK;
-  if (dtype == SR_DT_BF16)
-    k_act<bf16><<<M, 128, 0, st>>>(in, F, act, (bf16*)out);
-  else
-    k_act<float><<<M, 128, 0, st>>>(in, F, act, (float*)out);
+  SR_DISPATCH_ET(et, T, (k_act<T><<<M, 128, 0, st>>>(in, F, act, (T*)out)));
   SR_LAUNCH();
   return SR_OK;
 }
 
-sr_status launch_score_head(int dtype, int norm, const float* x, const int* rows, int n, const void* w,
-                            const void* b, float eps, const void* head, int d, float* rewards, cudaStream_t st) {
+sr_status launch_score_head(int et, int norm, const float* x, const int* rows, int n, const void* w, const void* b,
+                            float eps, const void* head, int d, float* rewards, cudaStream_t st) {
   if (n == 0) return SR_OK;
   const int ln = norm == SR_NORM_LAYER;
-  if (dtype == SR_DT_BF16)
-    k_score_head<bf16><<<n, threads_for(d), 0, st>>>(x, rows, (const bf16*)w, (const bf16*)b, eps, ln,
-                                                     (const bf16*)head, d, rewards);
-  else
-    k_score_head<float><<<n, threads_for(d), 0, st>>>(x, rows, (const float*)w, (const float*)b, eps, ln,
-                                                      (const float*)head, d, rewards);
+  SR_DISPATCH_ET(et, T, (k_score_head<T><<<n, threads_for(d), 0, st>>>(x, rows, (const T*)w, (const T*)b, eps, ln,
+                                                                       (const T*)head, d, rewards)));
   SR_LAUNCH();
   return SR_OK;
 }
 
-sr_status launch_copy_page(int dtype, void* pool, long long layer_stride, int n_layers, int page_elems, int src,
+sr_status launch_copy_page(int et, void* pool, long long layer_stride, int n_layers, int page_elems, int src,
                            const int* dst, int n_dst, cudaStream_t st) {
   if (n_dst == 0) return SR_OK;
   dim3 grid(n_dst, n_layers);
-  if (dtype == SR_DT_BF16)
-    k_copy_page<bf16><<<grid, 256, 0, st>>>((bf16*)pool, layer_stride, page_elems, src, dst);
-  else
-    k_copy_page<float><<<grid, 256, 0, st>>>((float*)pool, layer_stride, page_elems, src, dst);
+  SR_DISPATCH_ET(et, T, (k_copy_page<T><<<grid, 256, 0, st>>>((T*)pool, layer_stride, page_elems, src, dst)));
+  SR_LAUNCH();
+  return SR_OK;
+}
+
+sr_status launch_bf16_to_f16(void* p, size_t n, cudaStream_t st) {
+  if (n == 0) return SR_OK;
+  const size_t blocks = std::min<size_t>((n + 255) / 256, 65535 * 8);
+  k_bf16_to_f16<<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<uint16_t*>(p), n);
   SR_LAUNCH();
   return SR_OK;
 }

@@ -1,8 +1,9 @@
-// bf16 dense layers on the 5th-generation tensor cores (tcgen05 + TMEM + TMA), C = A W^T.
+// Dense layers on the 5th-generation tensor cores (tcgen05 + TMEM + TMA), C = A W^T, with A and W
+// both fp16 or both bf16 (kind::f16) and fp32 accumulation.
 //
 // Every projection of the generator and reward model (QKV, O, gate/up, down, LM head) is one
 // of these GEMMs (Section 4.2 generation and partial-reward scoring both run them; Section 3
-// defines the models).  A [M][K] and W [N][K] are K-major bf16; the accumulator is fp32 in
+// defines the models).  A [M][K] and W [N][K] are K-major 16-bit; the accumulator is fp32 in
 // tensor memory.
 //
 // Design (persistent, warp-specialised, one CTA per SM):
@@ -36,10 +37,12 @@ constexpr int BAR_BYTES = 256;
 constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
 constexpr unsigned long long WAIT_NS = 2000000000ull;
 
-// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1), B bf16
-// (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                           ((uint32_t)(BM >> 4) << 24);
+// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B format at bits 7-9 / 10-12
+// (0 = fp16, 1 = bf16), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_for(bool bf) {
+  return (1u << 4) | ((bf ? 1u : 0u) << 7) | ((bf ? 1u : 0u) << 10) | ((uint32_t)(BN >> 3) << 17) |
+         ((uint32_t)(BM >> 4) << 24);
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -97,11 +100,11 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t addr) {
   return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
           d_tmem),
-      "l"(a), "l"(b), "r"(IDESC), "r"(accumulate));
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
 }
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
@@ -130,14 +133,24 @@ __device__ __forceinline__ float gelu_f(float x) {
   return 0.5f * x * (1.f + tanhf(c * (x + 0.044715f * x * x * x)));
 }
 
-__device__ __forceinline__ void store_bf16x32(bf16* dst, const float* v) {
+// 32 consecutive outputs of one row as 16-bit values (bf16, or fp16 saturated at +-65504)
+__device__ __forceinline__ void store16x32(void* dst, const float* v, bool bf) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    __nv_bfloat162 h[4];
+    uint32_t w[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(v[q * 8 + 2 * j], v[q * 8 + 2 * j + 1]);
-    d4[q] = *reinterpret_cast<uint4*>(h);
+    for (int j = 0; j < 4; ++j) {
+      const float a = v[q * 8 + 2 * j], b = v[q * 8 + 2 * j + 1];
+      if (bf) {
+        __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+        w[j] = *reinterpret_cast<uint32_t*>(&h);
+      } else {
+        __half2 h = __floats2half2_rn(fminf(fmaxf(a, -65504.f), 65504.f), fminf(fmaxf(b, -65504.f), 65504.f));
+        w[j] = *reinterpret_cast<uint32_t*>(&h);
+      }
+    }
+    d4[q] = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
 
@@ -145,6 +158,7 @@ struct EpiArgs {
   void* out;
   int ldo;  // elements
   int kind;
+  int bf;   // operands and 16-bit outputs are bf16 (1) or fp16 (0)
 };
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -163,6 +177,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t idesc = idesc_for(ep.bf != 0);
   const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN, num_tiles = num_m * num_n;
   const int num_k = (K + BK - 1) / BK;
 
@@ -248,7 +263,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint64_t b0 = sdesc(smem_u32(sB + stage * B_BYTES));
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes per K=16 step inside the swizzle atom
-            umma(d_tmem, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), (kb | kk) != 0);
+            umma(d_tmem, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc, (kb | kk) != 0);
           umma_commit(&empty[stage]);
           if (++stage == STAGES) stage = 0, phase ^= 1u;
         }
@@ -296,8 +311,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (row < M && col0 + c < N) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) g[j] = (ep.kind == EPI_SWIGLU ? silu_f(g[j]) : gelu_f(g[j])) * u[j];
-            bf16* dst = reinterpret_cast<bf16*>(ep.out) + (size_t)row * ep.ldo + (col0 + c) / 2;
-            store_bf16x32(dst, g);
+            uint16_t* dst = reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + (col0 + c) / 2;
+            store16x32(dst, g, ep.bf != 0);
           }
         }
       } else {
@@ -323,7 +338,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
               }
-              store_bf16x32(reinterpret_cast<bf16*>(ep.out) + (size_t)row * ep.ldo + col0 + c, v);
+              store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col0 + c, v, ep.bf != 0);
             }
           }
         }
@@ -347,7 +362,7 @@ std::once_flag g_encode_once;
 int g_num_sms = 0;
 int* g_err = nullptr;
 
-sr_status encode_kmajor(CUtensorMap* map, const bf16* base, int rows, int K, int box_rows) {
+sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, int K, int box_rows) {
   std::call_once(g_encode_once, [] {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -361,7 +376,8 @@ sr_status encode_kmajor(CUtensorMap* map, const bf16* base, int rows, int K, int
   cuuint64_t strides[1] = {(cuuint64_t)K * 2};
   cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<bf16*>(base), dims, strides, box, estr,
+  CUresult r = g_encode(map, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
+                        const_cast<void*>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return set_err(SR_ERR_INVALID_ARG, "cuTensorMapEncodeTiled failed (%d)", (int)r);
@@ -370,7 +386,9 @@ sr_status encode_kmajor(CUtensorMap* map, const bf16* base, int rows, int K, int
 
 }  // namespace
 
-sr_status gemm_bf16(const bf16* A, const bf16* W, void* C, int M, int N, int K, int epi, cudaStream_t st) {
+sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, int K, int epi, cudaStream_t st) {
+  if (et != SR_DT_BF16 && et != SR_DT_F16) return set_err(SR_ERR_INVALID_ARG, "gemm: operands must be bf16 or fp16");
+  const bool bf = et == SR_DT_BF16;
   if (M <= 0 || N <= 0 || K <= 0) return M == 0 ? SR_OK : set_err(SR_ERR_INVALID_ARG, "gemm: bad shape");
   if (K % 8 != 0 || N % 32 != 0 || ((epi == EPI_SWIGLU || epi == EPI_GEGLU) && N % 64 != 0))
     return set_err(SR_ERR_INVALID_ARG, "gemm: needs K %% 8 == 0 and N %% 32 == 0 (N %% 64 for gated)");
@@ -385,9 +403,9 @@ sr_status gemm_bf16(const bf16* A, const bf16* W, void* C, int M, int N, int K, 
     SR_CUDA(cudaMemset(g_err, 0, sizeof(int)));
   }
   CUtensorMap ta, tb;
-  SR_TRY(encode_kmajor(&ta, A, M, K, BM));
-  SR_TRY(encode_kmajor(&tb, W, N, K, BN));
-  EpiArgs ep{C, (epi == EPI_SWIGLU || epi == EPI_GEGLU) ? N / 2 : N, epi};
+  SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
+  SR_TRY(encode_kmajor(&tb, W, bf, N, K, BN));
+  EpiArgs ep{C, (epi == EPI_SWIGLU || epi == EPI_GEGLU) ? N / 2 : N, epi, bf ? 1 : 0};
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = tiles < g_num_sms ? tiles : g_num_sms;
   k_gemm_tc<<<grid, NUM_THREADS, SMEM_BYTES, st>>>(ta, tb, ep, M, N, K, g_err);

@@ -142,6 +142,7 @@ struct LayerW {
 struct Model {
   sr_model_desc d{};
   int esz = 2;
+  int et = SR_DT_F16;  // device element type: SR_DT_F32 or SR_DT_F16
   char* blob = nullptr;
   void *tok_emb = nullptr, *pos_emb = nullptr, *final_w = nullptr, *final_b = nullptr, *lm_head = nullptr,
        *score_head = nullptr;
@@ -160,16 +161,17 @@ sr_status check_desc(const sr_model_desc* m, const char* who) {
   if (m->norm != SR_NORM_RMS && m->norm != SR_NORM_LAYER) return set_err(SR_ERR_INVALID_ARG, "%s: norm", who);
   if (m->act < SR_ACT_SWIGLU || m->act > SR_ACT_GEGLU) return set_err(SR_ERR_INVALID_ARG, "%s: act", who);
   if (m->pos != SR_POS_ROPE && m->pos != SR_POS_LEARNED) return set_err(SR_ERR_INVALID_ARG, "%s: pos", who);
-  if (m->dtype != SR_DT_F32 && m->dtype != SR_DT_BF16) return set_err(SR_ERR_INVALID_ARG, "%s: dtype", who);
+  if (m->dtype != SR_DT_F32 && m->dtype != SR_DT_BF16 && m->dtype != SR_DT_F16)
+    return set_err(SR_ERR_INVALID_ARG, "%s: dtype", who);
   if (m->n_heads % m->n_kv_heads) return set_err(SR_ERR_UNSUPPORTED, "%s: n_heads %% n_kv_heads != 0", who);
   if (m->head_dim % 2) return set_err(SR_ERR_UNSUPPORTED, "%s: odd head_dim", who);
   if (m->ffn_dim % 32) return set_err(SR_ERR_UNSUPPORTED, "%s: ffn_dim %% 32 != 0", who);
-  if (m->dtype == SR_DT_BF16) {
+  if (m->dtype != SR_DT_F32) {
     if (m->d_model % 64 || m->ffn_dim % 64 || m->vocab % 32 || (m->n_heads * m->head_dim) % 64)
-      return set_err(SR_ERR_UNSUPPORTED, "%s: bf16 needs d_model, ffn_dim, n_heads*head_dim %% 64 == 0 and vocab %% 32 == 0",
-                     who);
+      return set_err(SR_ERR_UNSUPPORTED,
+                     "%s: 16-bit models need d_model, ffn_dim, n_heads*head_dim %% 64 == 0 and vocab %% 32 == 0", who);
     if (m->head_dim != 32 && m->head_dim != 64 && m->head_dim != 128 && m->head_dim != 256)
-      return set_err(SR_ERR_UNSUPPORTED, "%s: head_dim %d (bf16 needs 32/64/128/256)", who, m->head_dim);
+      return set_err(SR_ERR_UNSUPPORTED, "%s: head_dim %d (16-bit models need 32/64/128/256)", who, m->head_dim);
   }
   return SR_OK;
 }
@@ -178,7 +180,8 @@ sr_status check_desc(const sr_model_desc* m, const char* who) {
 // device allocation; gate/up rows are interleaved in blocks of 32 for the fused GLU epilogue.
 sr_status load_model(Model& M, const sr_model_desc* d, const void* src) {
   M.d = *d;
-  M.esz = d->dtype == SR_DT_BF16 ? 2 : 4;
+  M.esz = d->dtype == SR_DT_F32 ? 4 : 2;
+  M.et = d->dtype == SR_DT_F32 ? SR_DT_F32 : SR_DT_F16;
   const size_t D = d->d_model, F = d->ffn_dim, V = d->vocab, E = M.esz;
   const bool ln = d->norm == SR_NORM_LAYER;
   struct T {
@@ -240,6 +243,7 @@ sr_status load_model(Model& M, const sr_model_desc* d, const void* src) {
     }
     soff += bytes;
   }
+  if (d->dtype == SR_DT_BF16) SR_TRY(launch_bf16_to_f16(M.blob, total / 2, 0));  // fp16 operands on the device
   if (d->pos == SR_POS_ROPE) {
     SR_CUDA(cudaMalloc(&M.rope, (size_t)d->max_pos * (d->head_dim / 2) * sizeof(float2)));
     SR_TRY(launch_rope_table(M.rope, d->max_pos, d->head_dim, (double)d->rope_theta, 0));
@@ -280,7 +284,7 @@ struct Work {
     SR_TRY(grow(v, c_v, R * m.kv_tok_elems() * E));
     SR_TRY(grow(att, c_att, R * HD * E));
     SR_TRY(grow(h, c_h, R * F * E));
-    if (m.d.dtype == SR_DT_F32) SR_TRY(grow(gu, c_gu, R * F * (m.gated() ? 2 : 1)));
+    if (m.et == SR_DT_F32) SR_TRY(grow(gu, c_gu, R * F * (m.gated() ? 2 : 1)));
     rows = n;
     return SR_OK;
   }
@@ -321,21 +325,20 @@ sr_status linear(const Model& m, const void* A, const void* W, void* C, int M, i
   const double out_b = (epi == EPI_F32) ? 4.0 * M * N : (epi == EPI_ADD_F32) ? 8.0 * M * N
                        : (epi == EPI_SWIGLU || epi == EPI_GEGLU) ? E * M * N / 2 : E * M * N;
   Scope sc(pf, cls, st, 2.0 * M * N * K, E * ((double)M * K + (double)N * K) + out_b);
-  if (m.d.dtype == SR_DT_BF16)
-    return gemm_bf16((const bf16*)A, (const bf16*)W, C, M, N, K, epi, st);
+  if (m.et == SR_DT_F16) return gemm_tc(SR_DT_F16, A, W, C, M, N, K, epi, st);
   return gemm_f32((const float*)A, (const float*)W, (float*)C, M, N, K, epi, st);
 }
 
 // MLP block: x += W_down act(W_gate h, W_up h) (or GELU(W_fc h)), h = Norm(x) already in w.xn
 sr_status mlp(const Model& m, Work& w, const LayerW& lw, int M, cudaStream_t st, Prof* pf, int cls) {
   const int D = m.d.d_model, F = m.d.ffn_dim;
-  if (m.d.dtype == SR_DT_BF16) {
+  if (m.et == SR_DT_F16) {
     const int epi = m.d.act == SR_ACT_SWIGLU ? EPI_SWIGLU : (m.d.act == SR_ACT_GEGLU ? EPI_GEGLU : EPI_GELU);
     SR_TRY(linear(m, w.xn, lw.wgu, w.h, M, m.gated() ? 2 * F : F, D, epi, st, pf, cls));
   } else {
     SR_TRY(linear(m, w.xn, lw.wgu, w.gu, M, m.gated() ? 2 * F : F, D, EPI_F32, st, pf, cls));
     Scope sc(pf, SR_KC_ELEMENTWISE, st);
-    SR_TRY(launch_act(m.d.dtype, m.d.act, w.gu, M, F, w.h, st));
+    SR_TRY(launch_act(m.et, m.d.act, w.gu, M, F, w.h, st));
   }
   return linear(m, w.h, lw.wdown, w.x, M, D, F, EPI_ADD_F32, st, pf, cls);
 }
@@ -349,13 +352,13 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
   SR_TRY(w.ensure(m, M));
   {
     Scope sc(pf, SR_KC_ELEMENTWISE, st);
-    SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, tok, pos, M, D, w.x, st));
+    SR_TRY(launch_embed(m.et, m.tok_emb, m.pos_emb, tok, pos, M, D, w.x, st));
   }
   for (int l = 0; l < d.n_layers; ++l) {
     const LayerW& lw = m.L[l];
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
-      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, M, D, w.xn, st));
+      SR_TRY(launch_norm(m.et, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, M, D, w.xn, st));
     }
     SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, M, m.qkv_dim(), D, EPI_F32, st, pf, gcls));
     char* kout = kv.store_k ? kv.store_k + l * kv.store_layer_bytes : w.k;
@@ -364,7 +367,7 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
     if (kv.pool) sink = KvSink{static_cast<char*>(kv.pool) + l * kv.pool_layer_bytes, kv.page_row, 0, nullptr};
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
-      SR_TRY(launch_rope_store(d.dtype, w.qkv, M, pos, m.rope, Hq, Hkv, dh, w.q, kout, vout, sink, st));
+      SR_TRY(launch_rope_store(m.et, w.qkv, M, pos, m.rope, Hq, Hkv, dh, w.q, kout, vout, sink, st));
     }
     const char* pk = plan.n_pre ? plan.pre_k + l * plan.pre_layer_bytes : nullptr;
     const char* pv = plan.n_pre ? plan.pre_v + l * plan.pre_layer_bytes : nullptr;
@@ -372,11 +375,10 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
     {
       Scope sa(pf, SR_KC_ATTN_PREFILL, st, attn_flops,
                2.0 * M * (double)Hq * dh * m.esz + 2.0 * kvb * (M + (double)plan.n_pre));
-      if (d.dtype == SR_DT_BF16)
-        SR_TRY(launch_prefill_attention((const bf16*)w.q, (const bf16*)kout, (const bf16*)vout, (const bf16*)pk,
-                                        (const bf16*)pv, plan.n_pre, plan.seq_off, plan.n_seq, plan.tile_seq,
-                                        plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window, (bf16*)w.att,
-                                        st));
+      if (m.et == SR_DT_F16)
+        SR_TRY(launch_prefill_attention(m.et, w.q, kout, vout, pk, pv, plan.n_pre, plan.seq_off, plan.n_seq,
+                                        plan.tile_seq, plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window,
+                                        w.att, st));
       else
         SR_TRY(launch_prefill_attention_f32((const float*)w.q, (const float*)kout, (const float*)vout,
                                             (const float*)pk, (const float*)pv, plan.n_pre, plan.seq_off, plan.n_seq,
@@ -385,7 +387,7 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
     SR_TRY(linear(m, w.att, lw.wo, w.x, M, D, Hq * dh, EPI_ADD_F32, st, pf, gcls));
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
-      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, M, D, w.xn, st));
+      SR_TRY(launch_norm(m.et, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, M, D, w.xn, st));
     }
     SR_TRY(mlp(m, w, lw, M, st, pf, gcls));
   }
@@ -589,7 +591,7 @@ sr_status prefill_prompt(sr_ctx* c, sr_batch& b) {
   // logits of the last prompt position (the distribution of token 0 of every candidate)
   {
     Scope sc(pf, SR_KC_ELEMENTWISE, c->st);
-    SR_TRY(launch_norm(g.d.dtype, g.d.norm, c->wg.x + (size_t)(P - 1) * g.d.d_model, g.final_w, g.final_b,
+    SR_TRY(launch_norm(g.et, g.d.norm, c->wg.x + (size_t)(P - 1) * g.d.d_model, g.final_w, g.final_b,
                        g.d.norm_eps, 1, g.d.d_model, c->wg.xn, c->st));
   }
   SR_TRY(linear(g, c->wg.xn, g.lm_head, c->logits0, 1, g.d.vocab, g.d.d_model, EPI_F32, c->st, pf,
@@ -608,7 +610,7 @@ sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
   }
   if (b.has_tail) {
     Scope sc(pf, SR_KC_ELEMENTWISE, c->st);
-    SR_TRY(launch_copy_page(g.d.dtype, c->pool, (long long)(pool_layer_bytes(c) / g.esz), g.d.n_layers,
+    SR_TRY(launch_copy_page(g.et, c->pool, (long long)(pool_layer_bytes(c) / g.esz), g.d.n_layers,
                             (int)c->page_elems, c->pool_cap_pages - 1, c->tail_dst, count, c->st));
   }
   {
@@ -655,36 +657,36 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
   const double attn_flops = 4.0 * n * Hq * dh * (double)eff_len;
   {
     Scope sc(pf, SR_KC_ELEMENTWISE, st);
-    SR_TRY(launch_embed(d.dtype, m.tok_emb, m.pos_emb, c->tok_in, c->pos_in, n, D, w.x, st));
+    SR_TRY(launch_embed(m.et, m.tok_emb, m.pos_emb, c->tok_in, c->pos_in, n, D, w.x, st));
   }
   for (int l = 0; l < d.n_layers; ++l) {
     const LayerW& lw = m.L[l];
     char* pool_l = c->pool + l * pool_layer_bytes(c);
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
-      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, n, D, w.xn, st));
+      SR_TRY(launch_norm(m.et, d.norm, w.x, lw.attn_w, lw.attn_b, d.norm_eps, n, D, w.xn, st));
     }
     SR_TRY(linear(m, w.xn, lw.wqkv, w.qkv, n, m.qkv_dim(), D, EPI_F32, st, pf, SR_KC_GEMM_DECODE));
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
-      SR_TRY(launch_rope_store(d.dtype, w.qkv, n, c->pos_in, m.rope, Hq, Hkv, dh, w.q, nullptr, nullptr,
+      SR_TRY(launch_rope_store(m.et, w.qkv, n, c->pos_in, m.rope, Hq, Hkv, dh, w.q, nullptr, nullptr,
                                KvSink{pool_l, c->pt, b.max_pages, c->live}, st));
     }
     {
       Scope sc(pf, SR_KC_ATTN_DECODE, st, attn_flops, attn_bytes);
-      SR_TRY(launch_decode_attention(d.dtype, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
+      SR_TRY(launch_decode_attention(m.et, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
                                      d.window, w.att, w.part, splits, st));
     }
     SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, st, pf, SR_KC_GEMM_DECODE));
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
-      SR_TRY(launch_norm(d.dtype, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, n, D, w.xn, st));
+      SR_TRY(launch_norm(m.et, d.norm, w.x, lw.mlp_w, lw.mlp_b, d.norm_eps, n, D, w.xn, st));
     }
     SR_TRY(mlp(m, w, lw, n, st, pf, SR_KC_GEMM_DECODE));
   }
   {
     Scope sc(pf, SR_KC_ELEMENTWISE, st);
-    SR_TRY(launch_norm(d.dtype, d.norm, w.x, m.final_w, m.final_b, d.norm_eps, n, D, w.xn, st));
+    SR_TRY(launch_norm(m.et, d.norm, w.x, m.final_w, m.final_b, d.norm_eps, n, D, w.xn, st));
   }
   SR_TRY(linear(m, w.xn, m.lm_head, c->logits, n, d.vocab, D, EPI_F32, st, pf, SR_KC_GEMM_DECODE));
   if (logits_host)
@@ -798,7 +800,7 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
                                   SR_KC_GEMM_SCORE, prefill_attn_flops(r, taus, ch.s0, ch.ns, b.P))) != SR_OK)
       break;
     Scope sc(&c->prof, SR_KC_ELEMENTWISE, c->st);
-    if ((status = launch_score_head(r.d.dtype, r.d.norm, c->wr.x, c->last_row, ch.ns, r.final_w, r.final_b,
+    if ((status = launch_score_head(r.et, r.d.norm, c->wr.x, c->last_row, ch.ns, r.final_w, r.final_b,
                                     r.d.norm_eps, r.score_head, r.d.d_model, rewards_dev + ch.s0, c->st)) != SR_OK)
       break;
   }
@@ -991,7 +993,8 @@ sr_status sr_init(sr_ctx** out, const sr_model_desc* gen, const void* gen_w, con
   if (!gen_w || !rm_w) return set_err(SR_ERR_INVALID_ARG, "null weights");
   if (!gen->has_lm_head) return set_err(SR_ERR_INVALID_ARG, "generator needs an LM head");
   if (!rm->has_scalar_head) return set_err(SR_ERR_INVALID_ARG, "reward model needs a scalar head");
-  if (gen->dtype != rm->dtype) return set_err(SR_ERR_INVALID_ARG, "generator and reward model dtypes differ");
+  if ((gen->dtype == SR_DT_F32) != (rm->dtype == SR_DT_F32))
+    return set_err(SR_ERR_INVALID_ARG, "generator and reward model must both be fp32 or both 16-bit");
   if (gen->vocab != rm->vocab) return set_err(SR_ERR_INVALID_ARG, "generator and reward model vocabularies differ");
   if (page_tokens != PAGE) return set_err(SR_ERR_INVALID_ARG, "page_tokens must be 16");
   int ndev = 0;
@@ -1221,7 +1224,7 @@ sr_status sr_k_gemm(int dtype, const void* A, const void* W, void* C, int M, int
   if (!A || !W || !C) return set_err(SR_ERR_INVALID_ARG, "sr_k_gemm: null argument");
   if (epilogue < 0 || epilogue > EPI_GELU) return set_err(SR_ERR_INVALID_ARG, "sr_k_gemm: bad epilogue");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (dtype == SR_DT_BF16) return gemm_bf16((const bf16*)A, (const bf16*)W, C, M, N, K, epilogue, st);
+  if (dtype == SR_DT_BF16 || dtype == SR_DT_F16) return gemm_tc(dtype, A, W, C, M, N, K, epilogue, st);
   if (dtype == SR_DT_F32) return gemm_f32((const float*)A, (const float*)W, (float*)C, M, N, K, epilogue, st);
   return set_err(SR_ERR_INVALID_ARG, "sr_k_gemm: bad dtype");
 }
@@ -1247,9 +1250,9 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
   return s;
 }
 
-sr_status sr_k_prefill_attention(const void* q, const void* k, const void* v, const void* k_pre, const void* v_pre,
-                                 int n_pre, const int32_t* seq_off, int n_seq, int pos0, int n_heads, int n_kv_heads,
-                                 int head_dim, int window, void* out, void* stream) {
+sr_status sr_k_prefill_attention(int dtype, const void* q, const void* k, const void* v, const void* k_pre,
+                                 const void* v_pre, int n_pre, const int32_t* seq_off, int n_seq, int pos0,
+                                 int n_heads, int n_kv_heads, int head_dim, int window, void* out, void* stream) {
   if (!q || !k || !v || !seq_off || !out || n_seq < 1) return set_err(SR_ERR_INVALID_ARG, "null argument");
   if (n_pre > 0 && (!k_pre || !v_pre)) return set_err(SR_ERR_INVALID_ARG, "prefix pointers missing");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1265,9 +1268,8 @@ sr_status sr_k_prefill_attention(const void* q, const void* k, const void* v, co
   std::vector<int> hcat(ts);
   hcat.insert(hcat.end(), tq.begin(), tq.end());
   SR_CUDA(cudaMemcpyAsync(d, hcat.data(), 2 * nt * sizeof(int), cudaMemcpyHostToDevice, st));
-  sr_status s = launch_prefill_attention((const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)k_pre,
-                                         (const bf16*)v_pre, n_pre, seq_off, n_seq, d, d + nt, nt, pos0, n_heads,
-                                         n_kv_heads, head_dim, window, (bf16*)out, st);
+  sr_status s = launch_prefill_attention(dtype, q, k, v, k_pre, v_pre, n_pre, seq_off, n_seq, d, d + nt, nt, pos0,
+                                         n_heads, n_kv_heads, head_dim, window, out, st);
   cudaStreamSynchronize(st);  // the host copy of the tile list must outlive the upload
   cudaFreeAsync(d, st);
   return s;

@@ -19,7 +19,7 @@ import torch
 
 from . import binding as sr
 
-DT_BF16 = 1
+DT_F16 = 2
 
 
 def _time(fn, iters=20, warm=3):
@@ -38,12 +38,12 @@ def _time(fn, iters=20, warm=3):
 
 def gemm(M, N, K, epi=0, iters=20):
     g = torch.Generator(device="cuda").manual_seed(0)
-    A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
-    W = torch.randn(N, K, device="cuda", generator=g).to(torch.bfloat16)
+    A = torch.randn(M, K, device="cuda", generator=g).to(torch.float16)
+    W = torch.randn(N, K, device="cuda", generator=g).to(torch.float16)
     C = torch.zeros(M, N // 2 if epi in (3, 4) else N, device="cuda",
-                    dtype=torch.float32 if epi in (0, 1) else torch.bfloat16)
+                    dtype=torch.float32 if epi in (0, 1) else torch.float16)
     s = torch.cuda.current_stream().cuda_stream
-    ms = _time(lambda: sr.sr_k_gemm(DT_BF16, A, W, C, M, N, K, epi, s), iters)
+    ms = _time(lambda: sr.sr_k_gemm(DT_F16, A, W, C, M, N, K, epi, s), iters)
     fl = 2.0 * M * N * K
     by = 2.0 * (M * K + N * K) + C.numel() * C.element_size()
     return dict(kernel="gemm", M=M, N=N, K=K, epi=epi, ms=ms, tflops=fl / ms / 1e9, gbs=by / ms / 1e6)
@@ -51,14 +51,14 @@ def gemm(M, N, K, epi=0, iters=20):
 
 def decode_attn(b, Hq, Hkv, dh, L, iters=20):
     pages = (L + 15) // 16
-    pool = torch.randn(b * pages + 1, 2, Hkv, 16, dh, device="cuda").to(torch.bfloat16)
+    pool = torch.randn(b * pages + 1, 2, Hkv, 16, dh, device="cuda").to(torch.float16)
     pt = torch.randperm(b * pages, device="cuda").to(torch.int32).reshape(b, pages)
     ids = torch.arange(b, device="cuda", dtype=torch.int32)
     lens = torch.full((b,), L, device="cuda", dtype=torch.int32)
-    q = torch.randn(b, Hq, dh, device="cuda").to(torch.bfloat16)
+    q = torch.randn(b, Hq, dh, device="cuda").to(torch.float16)
     out = torch.zeros_like(q)
     s = torch.cuda.current_stream().cuda_stream
-    ms = _time(lambda: sr.sr_k_decode_attention(DT_BF16, q, pool, pt, pages, ids, lens, b, Hq, Hkv, dh, 0, out, s),
+    ms = _time(lambda: sr.sr_k_decode_attention(DT_F16, q, pool, pt, pages, ids, lens, b, Hq, Hkv, dh, 0, out, s),
                iters)
     by = b * L * Hkv * dh * 2 * 2 + 2 * q.numel() * 2
     return dict(kernel="decode_attn", b=b, Hq=Hq, Hkv=Hkv, dh=dh, len=L, ms=ms, gbs=by / ms / 1e6)
@@ -66,15 +66,15 @@ def decode_attn(b, Hq, Hkv, dh, L, iters=20):
 
 def prefill_attn(n_seq, tau, n_pre, Hq, Hkv, dh, iters=10):
     rows = n_seq * tau
-    q = torch.randn(rows, Hq, dh, device="cuda").to(torch.bfloat16)
-    k = torch.randn(rows, Hkv, dh, device="cuda").to(torch.bfloat16)
-    v = torch.randn(rows, Hkv, dh, device="cuda").to(torch.bfloat16)
-    kp = torch.randn(max(n_pre, 1), Hkv, dh, device="cuda").to(torch.bfloat16)
-    vp = torch.randn(max(n_pre, 1), Hkv, dh, device="cuda").to(torch.bfloat16)
+    q = torch.randn(rows, Hq, dh, device="cuda").to(torch.float16)
+    k = torch.randn(rows, Hkv, dh, device="cuda").to(torch.float16)
+    v = torch.randn(rows, Hkv, dh, device="cuda").to(torch.float16)
+    kp = torch.randn(max(n_pre, 1), Hkv, dh, device="cuda").to(torch.float16)
+    vp = torch.randn(max(n_pre, 1), Hkv, dh, device="cuda").to(torch.float16)
     off = torch.arange(0, rows + 1, tau, device="cuda", dtype=torch.int32)
     out = torch.zeros_like(q)
     s = torch.cuda.current_stream().cuda_stream
-    ms = _time(lambda: sr.sr_k_prefill_attention(q, k, v, kp, vp, n_pre, off, n_seq, n_pre, Hq, Hkv, dh, 0, out, s),
+    ms = _time(lambda: sr.sr_k_prefill_attention(DT_F16, q, k, v, kp, vp, n_pre, off, n_seq, n_pre, Hq, Hkv, dh, 0, out, s),
                iters)
     fl = 4.0 * Hq * dh * n_seq * (tau * n_pre + tau * (tau + 1) / 2)
     return dict(kernel="prefill_attn", n_seq=n_seq, tau=tau, n_pre=n_pre, ms=ms, tflops=fl / ms / 1e9)

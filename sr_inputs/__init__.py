@@ -24,7 +24,7 @@ import numpy as np
 NORM_RMS, NORM_LAYER = 0, 1
 ACT_SWIGLU, ACT_GELU, ACT_GEGLU = 0, 1, 2
 POS_ROPE, POS_LEARNED = 0, 1
-DT_F32, DT_BF16 = 0, 1
+DT_F32, DT_BF16, DT_F16 = 0, 1, 2
 SCHED_FIXED, SCHED_POOL_FULL = 0, 1
 
 

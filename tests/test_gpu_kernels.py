@@ -95,41 +95,47 @@ def _bf16(x):
     return torch.from_numpy(x).to(torch.bfloat16)
 
 
+T16 = {si.DT_BF16: torch.bfloat16, si.DT_F16: torch.float16}
+
+
+@pytest.mark.parametrize("dt", [si.DT_F16, si.DT_BF16])
 @pytest.mark.parametrize("M,N,K", [(1, 256, 64), (7, 512, 128), (130, 2304, 768), (300, 288, 1000), (257, 96, 520),
                                    (1024, 4096, 4096), (1, 32000, 768), (2048, 512, 64)])
-def test_gemm_bf16_fp32_out(sr, M, N, K):
+def test_gemm_tc_fp32_out(sr, dt, M, N, K):
     g = torch.Generator().manual_seed(M * 7 + N + K)
-    A = torch.randn(M, K, generator=g).to(torch.bfloat16)
-    W = torch.randn(N, K, generator=g).to(torch.bfloat16)
+    A = torch.randn(M, K, generator=g).to(T16[dt])
+    W = torch.randn(N, K, generator=g).to(T16[dt])
     ref = A.float() @ W.float().T
     C = torch.zeros(M, N, device="cuda")
-    sr.sr_k_gemm(si.DT_BF16, A.cuda(), W.cuda(), C, M, N, K, 0)
+    sr.sr_k_gemm(dt, A.cuda(), W.cuda(), C, M, N, K, 0)
     torch.testing.assert_close(C.cpu(), ref, rtol=2e-4, atol=2e-4 * np.sqrt(K))
     # epilogue 1: accumulate into the fp32 output (residual add)
     base = torch.randn(M, N, generator=g)
     C = base.cuda().clone()
-    sr.sr_k_gemm(si.DT_BF16, A.cuda(), W.cuda(), C, M, N, K, 1)
+    sr.sr_k_gemm(dt, A.cuda(), W.cuda(), C, M, N, K, 1)
     torch.testing.assert_close(C.cpu(), base + ref, rtol=2e-4, atol=2e-4 * np.sqrt(K))
 
 
+@pytest.mark.parametrize("dt", [si.DT_F16, si.DT_BF16])
 @pytest.mark.parametrize("epi", [2, 3, 4, 5])
 @pytest.mark.parametrize("M,N,K", [(5, 256, 64), (200, 1024, 512), (129, 512, 4096)])
-def test_gemm_bf16_epilogues(sr, epi, M, N, K):
+def test_gemm_tc_epilogues(sr, dt, epi, M, N, K):
     g = torch.Generator().manual_seed(epi * 1000 + M)
-    A = (torch.randn(M, K, generator=g) / np.sqrt(K)).to(torch.bfloat16)
-    W = torch.randn(N, K, generator=g).to(torch.bfloat16)
+    A = (torch.randn(M, K, generator=g) / np.sqrt(K)).to(T16[dt])
+    W = torch.randn(N, K, generator=g).to(T16[dt])
     acc = A.float() @ W.float().T
     if epi in (3, 4):
         blk = acc.reshape(M, N // 64, 2, 32)
         gate, up = blk[:, :, 0, :].reshape(M, N // 2), blk[:, :, 1, :].reshape(M, N // 2)
         act = torch.nn.functional.silu(gate) if epi == 3 else torch.nn.functional.gelu(gate, approximate="tanh")
         ref = act * up
-        C = torch.zeros(M, N // 2, dtype=torch.bfloat16, device="cuda")
+        C = torch.zeros(M, N // 2, dtype=T16[dt], device="cuda")
     else:
         ref = acc if epi == 2 else torch.nn.functional.gelu(acc, approximate="tanh")
-        C = torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
-    sr.sr_k_gemm(si.DT_BF16, A.cuda(), W.cuda(), C, M, N, K, epi)
-    torch.testing.assert_close(C.float().cpu(), ref.to(torch.bfloat16).float(), rtol=1.6e-2, atol=1e-3)
+        C = torch.zeros(M, N, dtype=T16[dt], device="cuda")
+    sr.sr_k_gemm(dt, A.cuda(), W.cuda(), C, M, N, K, epi)
+    tol = 1.6e-2 if dt == si.DT_BF16 else 2e-3
+    torch.testing.assert_close(C.float().cpu(), ref.to(T16[dt]).float(), rtol=tol, atol=1e-3)
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 64, 16), (33, 200, 77), (128, 512, 128)])
@@ -143,14 +149,17 @@ def test_gemm_f32(sr, M, N, K):
 
 
 # ------------------------------------------------------------------------------------------ attention
-def _round_bf16(x):
-    return torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+def _round16(x, dt=si.DT_F16):
+    return torch.from_numpy(x).to(T16[dt]).float().numpy()
 
 
 @pytest.mark.parametrize("dt,Hq,Hkv,dh,window,lens", [
-    (si.DT_BF16, 32, 8, 128, 0, [1, 15, 16, 17, 300, 511, 512, 513, 1100, 2000]),
-    (si.DT_BF16, 12, 12, 64, 0, [5, 129, 700]),
-    (si.DT_BF16, 32, 8, 128, 100, [50, 100, 101, 900]),
+    (si.DT_F16, 32, 8, 128, 0, [1, 15, 16, 17, 300, 511, 512, 513, 1100, 2000]),
+    (si.DT_F16, 12, 12, 64, 0, [5, 129, 700]),
+    (si.DT_F16, 32, 8, 128, 100, [50, 100, 101, 900]),
+    (si.DT_F16, 16, 2, 128, 0, [33, 64, 600]),
+    (si.DT_F16, 4, 4, 32, 0, [1, 16, 33, 80]),
+    (si.DT_BF16, 32, 8, 128, 0, [7, 300, 1300]),
     (si.DT_F32, 4, 4, 32, 0, [1, 16, 33, 80]),
 ])
 def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens):
@@ -160,12 +169,12 @@ def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens):
     n_pages = b * max_pages + 3
     pool = rng.standard_normal((n_pages, 2, Hkv, 16, dh)).astype(np.float32)
     q = rng.standard_normal((b, Hq, dh)).astype(np.float32)
-    if dt == si.DT_BF16:
-        pool, q = _round_bf16(pool), _round_bf16(q)
+    if dt != si.DT_F32:
+        pool, q = _round16(pool, dt), _round16(q, dt)
     perm = rng.permutation(n_pages).astype(np.int32)
     ids = rng.permutation(b).astype(np.int32)                       # slot s serves candidate ids[s]
     pt = perm[: b * max_pages].reshape(b, max_pages)                # page table indexed by candidate id
-    tdt = torch.bfloat16 if dt == si.DT_BF16 else torch.float32
+    tdt = T16.get(dt, torch.float32)
     out = torch.zeros(b, Hq, dh, dtype=tdt, device="cuda")
     sr.sr_k_decode_attention(dt, dev(q, tdt), dev(pool, tdt), dev(pt), max_pages, dev(ids),
                              dev(np.array(lens, np.int32)), b, Hq, Hkv, dh, window, out)
@@ -176,30 +185,31 @@ def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens):
         K = pool[pages, 0].transpose(0, 2, 1, 3).reshape(-1, Hkv, dh)[:L]
         Vv = pool[pages, 1].transpose(0, 2, 1, 3).reshape(-1, Hkv, dh)[:L]
         want = otr.attention(q[s][None, None], K[None], Vv[None], np.array([[L - 1]]), np.arange(L)[None], window)
-        tol = 1e-2 if dt == si.DT_BF16 else 2e-5
+        tol = {si.DT_BF16: 1e-2, si.DT_F16: 2e-3, si.DT_F32: 2e-5}[dt]
         np.testing.assert_allclose(got[s], want[0, 0], rtol=tol, atol=tol)
 
 
-@pytest.mark.parametrize("Hq,Hkv,dh,n_pre,taus,window", [
-    (32, 8, 128, 288, [1, 64, 65, 200, 7], 0),
-    (12, 12, 64, 128, [64, 3, 130], 0),
-    (8, 8, 256, 100, [70, 1, 128], 0),
-    (4, 2, 128, 0, [300], 0),
-    (8, 4, 64, 40, [90, 33], 50),
+@pytest.mark.parametrize("dt,Hq,Hkv,dh,n_pre,taus,window", [
+    (si.DT_F16, 32, 8, 128, 288, [1, 64, 65, 200, 7], 0),
+    (si.DT_F16, 12, 12, 64, 128, [64, 3, 130], 0),
+    (si.DT_F16, 8, 8, 256, 100, [70, 1, 128], 0),
+    (si.DT_F16, 4, 2, 128, 0, [300], 0),
+    (si.DT_F16, 8, 4, 64, 40, [90, 33], 50),
+    (si.DT_BF16, 32, 8, 128, 288, [1, 64, 65, 200, 7], 0),
 ])
-def test_prefill_attention(sr, Hq, Hkv, dh, n_pre, taus, window):
+def test_prefill_attention(sr, dt, Hq, Hkv, dh, n_pre, taus, window):
     rng = np.random.default_rng(dh + n_pre)
     rows = sum(taus)
-    q = _round_bf16(rng.standard_normal((rows, Hq, dh)).astype(np.float32))
-    k = _round_bf16(rng.standard_normal((rows, Hkv, dh)).astype(np.float32))
-    v = _round_bf16(rng.standard_normal((rows, Hkv, dh)).astype(np.float32))
-    kp = _round_bf16(rng.standard_normal((max(n_pre, 1), Hkv, dh)).astype(np.float32))
-    vp = _round_bf16(rng.standard_normal((max(n_pre, 1), Hkv, dh)).astype(np.float32))
+    q = _round16(rng.standard_normal((rows, Hq, dh)).astype(np.float32), dt)
+    k = _round16(rng.standard_normal((rows, Hkv, dh)).astype(np.float32), dt)
+    v = _round16(rng.standard_normal((rows, Hkv, dh)).astype(np.float32), dt)
+    kp = _round16(rng.standard_normal((max(n_pre, 1), Hkv, dh)).astype(np.float32), dt)
+    vp = _round16(rng.standard_normal((max(n_pre, 1), Hkv, dh)).astype(np.float32), dt)
     off = np.concatenate([[0], np.cumsum(taus)]).astype(np.int32)
     pos0 = n_pre
-    out = torch.zeros(rows, Hq, dh, dtype=torch.bfloat16, device="cuda")
-    b16 = torch.bfloat16
-    sr.sr_k_prefill_attention(dev(q, b16), dev(k, b16), dev(v, b16), dev(kp, b16), dev(vp, b16), n_pre, dev(off),
+    t = T16[dt]
+    out = torch.zeros(rows, Hq, dh, dtype=t, device="cuda")
+    sr.sr_k_prefill_attention(dt, dev(q, t), dev(k, t), dev(v, t), dev(kp, t), dev(vp, t), n_pre, dev(off),
                               len(taus), pos0, Hq, Hkv, dh, window, out)
     got = out.float().cpu().numpy()
     for j, t in enumerate(taus):
@@ -208,4 +218,5 @@ def test_prefill_attention(sr, Hq, Hkv, dh, n_pre, taus, window):
         V = np.concatenate([vp[:n_pre], v[sl]])
         kpos = np.concatenate([np.arange(n_pre), pos0 + np.arange(t)])
         want = otr.attention(q[sl][None], K[None], V[None], (pos0 + np.arange(t))[None], kpos[None], window)
-        np.testing.assert_allclose(got[sl], want[0], rtol=2e-2, atol=2e-2)
+        tol = 2e-2 if dt == si.DT_BF16 else 3e-3
+        np.testing.assert_allclose(got[sl], want[0], rtol=tol, atol=tol)
