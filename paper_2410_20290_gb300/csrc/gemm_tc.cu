@@ -7,19 +7,22 @@
 // tensor memory.
 //
 // Design (persistent, warp-specialised, one CTA per SM):
-//   warp 0      : TMA producer -- 128x64 A and 256x64 W tiles, 128-byte swizzle, STAGES-deep ring
-//   warp 1      : allocates 512 TMEM columns; one elected lane issues tcgen05.mma (M=128, N=256,
+//   warp 0      : TMA producer -- 128x64 A and BNx64 W tiles (BN = 256, 128 or 64, chosen per
+//                 shape so the tile count fills the SMs), 128-byte swizzle, STAGES-deep ring
+//                 (~192 KB of shared memory in flight per SM)
+//   warp 1      : allocates 2*BN TMEM columns; one elected lane issues tcgen05.mma (M=128, N=BN,
 //                 K=16) and tcgen05.commit to release smem stages / publish accumulators
 //   warps 2..5  : epilogue -- tcgen05.ld 32 lanes x 32 columns per warp (the warp's TMEM lane
 //                 quadrant is warp % 4), fused conversion / residual add / gated activation,
 //                 direct global stores
-// Two 256-column accumulators let the epilogue of tile i overlap the mainloop of tile i+1.
+// Two BN-column accumulators let the epilogue of tile i overlap the mainloop of tile i+1.
 // Tiles are walked M-fastest so that the CTAs running at the same time share W tiles in L2.
 // Every mbarrier wait is bounded (about 2 s of %globaltimer); on expiry the CTA records an error,
 // drains its own TMA copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
 #include <mutex>
 
 #include "common.cuh"
@@ -27,19 +30,24 @@
 namespace sr {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int BM = 128, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
-constexpr int B_BYTES = BN * BK * 2;  // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int NUM_THREADS = 192;
-constexpr int TMEM_COLS = 512;
 constexpr int BAR_BYTES = 256;
-constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
 constexpr unsigned long long WAIT_NS = 2000000000ull;
+
+template <int BN>
+struct Cfg {
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = (192 * 1024) / STAGE_BYTES;  // 4 / 6 / 8 stages for BN 256 / 128 / 64
+  static constexpr int TMEM_COLS = 2 * BN;                   // two accumulators
+  static constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
+};
 
 // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B format at bits 7-9 / 10-12
 // (0 = fp16, 1 = bf16), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-__host__ __device__ constexpr uint32_t idesc_for(bool bf) {
+__host__ __device__ constexpr uint32_t idesc_for(bool bf, int BN) {
   return (1u << 4) | ((bf ? 1u : 0u) << 7) | ((bf ? 1u : 0u) << 10) | ((uint32_t)(BN >> 3) << 17) |
          ((uint32_t)(BM >> 4) << 24);
 }
@@ -161,9 +169,12 @@ struct EpiArgs {
   int bf;   // operands and 16-bit outputs are bf16 (1) or fp16 (0)
 };
 
+template <int BN>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
               int N, int K, int* err) {
+  constexpr int B_BYTES = Cfg<BN>::B_BYTES, STAGE_BYTES = Cfg<BN>::STAGE_BYTES, STAGES = Cfg<BN>::STAGES;
+  constexpr int TMEM_COLS = Cfg<BN>::TMEM_COLS;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -177,7 +188,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t idesc = idesc_for(ep.bf != 0);
+  const uint32_t idesc = idesc_for(ep.bf != 0, BN);
   const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN, num_tiles = num_m * num_n;
   const int num_k = (K + BK - 1) / BK;
 
@@ -360,7 +371,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 int g_num_sms = 0;
+int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
 int* g_err = nullptr;
+
+// Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost, the cost
+// growing with BN (MMA and W-tile bytes) plus a fixed part (the A tile and the pipeline fill).
+int pick_bn(int M, int N) {
+  if (g_bn_override == 64 || g_bn_override == 128 || g_bn_override == 256) return g_bn_override;
+  int best = 256;
+  long long best_cost = -1;
+  for (int bn : {256, 128, 64}) {
+    const long long tiles = (long long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
+    const long long waves = (tiles + g_num_sms - 1) / g_num_sms;
+    const long long cost = waves * (bn + 64);
+    if (best_cost < 0 || cost < best_cost) best_cost = cost, best = bn;
+  }
+  return best;
+}
+
+template <int BN>
+sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
+                    cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::SMEM_BYTES));
+    attr = true;
+  }
+  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
+  k_gemm_tc<BN><<<grid, NUM_THREADS, Cfg<BN>::SMEM_BYTES, st>>>(ta, tb, ep, M, N, K, g_err);
+  SR_LAUNCH();
+  return SR_OK;
+}
 
 sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, int K, int box_rows) {
   std::call_once(g_encode_once, [] {
@@ -398,19 +440,19 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     int dev;
     SR_CUDA(cudaGetDevice(&dev));
     SR_CUDA(cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev));
-    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
     SR_CUDA(cudaMalloc(&g_err, sizeof(int)));
     SR_CUDA(cudaMemset(g_err, 0, sizeof(int)));
+    if (const char* e = getenv("SR_GEMM_BN")) g_bn_override = atoi(e);
   }
+  const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
+  const int bn = pick_bn(M, N);
   CUtensorMap ta, tb;
   SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
-  SR_TRY(encode_kmajor(&tb, W, bf, N, K, BN));
-  EpiArgs ep{C, (epi == EPI_SWIGLU || epi == EPI_GEGLU) ? N / 2 : N, epi, bf ? 1 : 0};
-  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
-  k_gemm_tc<<<grid, NUM_THREADS, SMEM_BYTES, st>>>(ta, tb, ep, M, N, K, g_err);
-  SR_LAUNCH();
-  return SR_OK;
+  SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn));
+  EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
+  if (bn == 64) return launch_bn<64>(ta, tb, ep, M, N, K, st);
+  if (bn == 128) return launch_bn<128>(ta, tb, ep, M, N, K, st);
+  return launch_bn<256>(ta, tb, ep, M, N, K, st);
 }
 
 // Device error word of the tensor-core GEMM (nonzero after a bounded wait expired).
