@@ -260,6 +260,24 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
                                 const int32_t* orig_ids, const int32_t* lens, int b, int n_heads, int n_kv_heads,
                                 int head_dim, int window, void* out, void* stream);
 
+/* sr_k_decode_attention_static -- the same decode attention for callers that cannot allocate
+ * device memory when they call (a server that has reserved all GPU memory up front, an
+ * allocator-free embedding, a caller holding a lock an allocation could block on).  The paper has
+ * no counterpart; this is an interface convenience.  Instead of a per-call buffer, the split
+ * partials (needed when a context exceeds 512 positions) use one fixed 8 MiB device array that
+ * every GPU loading the library holds until exit; the call allocates nothing.
+ *   max_len : an upper bound on lens[] (sizes the number of 512-position splits).
+ * Rejects, with SR_ERR_INVALID_ARG and a message, shapes needing more than 2^21 scratch floats
+ * (b * n_heads * splits * (head_dim + 2)).  The first call on a device looks up the array's device
+ * address (cudaGetSymbolAddress) with that device current; make that first call before any stream
+ * capture.  All calls share the array and it keeps the last call's contents (every value a call
+ * reads it has written itself, so nothing needs clearing); calls that overlap on the GPU, e.g. on
+ * two streams, race on it. */
+sr_status sr_k_decode_attention_static(int dtype, const void* q, const void* pool, const int32_t* page_table,
+                                       int pt_stride, const int32_t* orig_ids, const int32_t* lens, int b,
+                                       int n_heads, int n_kv_heads, int head_dim, int window, int max_len, void* out,
+                                       void* stream);
+
 /* Causal prefill attention over packed variable-length sequences with an
  * optional shared prefix.  Sequence j owns query/key rows seq_off[j] ..
  * seq_off[j+1]-1 of q [rows][n_heads][dh] and k, v [rows][n_kv][dh], at positions

@@ -90,6 +90,7 @@ _SIG = {
     "sr_k_rcut": [_P, _I, _F, _I, _P, _P, _P],
     "sr_k_gemm": [_I, _P, _P, _P, _I, _I, _I, _I, _P],
     "sr_k_decode_attention": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P, _P],
+    "sr_k_decode_attention_static": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P],
     "sr_k_prefill_attention": [_I, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _P, _P],
 }
 
@@ -271,6 +272,14 @@ def sr_k_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens,
     _check(LIB.sr_k_decode_attention(dtype, _ptr(q), _ptr(pool), _ptr(page_table), pt_stride, _ptr(orig_ids),
                                      _ptr(lens), b, n_heads, n_kv_heads, head_dim, window, _ptr(out),
                                      _stream(stream)))
+
+
+def sr_k_decode_attention_static(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
+                                 head_dim, window, max_len, out, stream=None):
+    """Decode attention that allocates nothing (split partials in the library's fixed device array)."""
+    _check(LIB.sr_k_decode_attention_static(dtype, _ptr(q), _ptr(pool), _ptr(page_table), pt_stride, _ptr(orig_ids),
+                                            _ptr(lens), b, n_heads, n_kv_heads, head_dim, window, max_len, _ptr(out),
+                                            _stream(stream)))
 
 
 def sr_k_prefill_attention(dtype, q, k, v, k_pre, v_pre, n_pre, seq_off, n_seq, pos0, n_heads, n_kv_heads, head_dim,

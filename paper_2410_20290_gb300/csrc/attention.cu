@@ -15,6 +15,7 @@
 // shared prefix (the prompt's KV) -- 64 query rows x one head per CTA, 64-key blocks staged by
 // cp.async, bf16 mma.sync m16n8k16 with fp32 accumulation, online softmax in registers.
 #include <algorithm>
+#include <mutex>
 #include <type_traits>
 
 #include "common.cuh"
@@ -764,3 +765,67 @@ sr_status launch_prefill_attention(int et, const void* q, const void* k, const v
 }
 
 }  // namespace sr
+
+// -------------------------------------------------------------------------------------------------
+// Decode attention without allocation.
+//
+// Some callers cannot allocate device memory at call time: code running inside a pre-sized memory
+// budget (an inference server that reserves all of the GPU's memory up front), allocator-free
+// embeddings, or callers holding locks under which an allocation could block.  For them the split
+// partials of decode attention live in this fixed device array instead of a buffer allocated per
+// call.  Every GPU that loads the library holds the array (8 MiB) until the process exits.
+// -------------------------------------------------------------------------------------------------
+namespace sr {
+namespace {
+
+constexpr size_t kStaticPartFloats = (size_t)1 << 21;  // 8 MiB of fp32 split partials
+static __device__ __align__(256) float g_static_part[kStaticPartFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+float* g_static_ptr[kMaxDevices] = {};  // device address of g_static_part, per device ordinal
+
+// In host code `g_static_part` names a host-side stand-in, not device memory, so its device
+// address is looked up once per device (with that device current) and cached.
+sr_status static_part_ptr(float** out) {
+  int dev = 0;
+  SR_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return set_err(SR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_part);
+    if (e != cudaSuccess)
+      return set_err(SR_ERR_CUDA, "cudaGetSymbolAddress(static decode-attention scratch): %s", cudaGetErrorString(e));
+    g_static_ptr[dev] = static_cast<float*>(p);
+  }
+  *out = g_static_ptr[dev];
+  return SR_OK;
+}
+
+}  // namespace
+}  // namespace sr
+
+extern "C" sr_status sr_k_decode_attention_static(int dtype, const void* q, const void* pool,
+                                                  const int32_t* page_table, int pt_stride, const int32_t* orig_ids,
+                                                  const int32_t* lens, int b, int n_heads, int n_kv_heads,
+                                                  int head_dim, int window, int max_len, void* out, void* stream) {
+  using namespace sr;
+  if (!q || !pool || !page_table || !orig_ids || !lens || !out)
+    return set_err(SR_ERR_INVALID_ARG, "sr_k_decode_attention_static: null argument");
+  if (b < 0 || n_kv_heads < 1 || n_heads < 1 || head_dim < 1 || max_len < 1)
+    return set_err(SR_ERR_INVALID_ARG, "sr_k_decode_attention_static: bad shape");
+  const int splits = decode_attention_max_splits(window > 0 ? std::min(max_len, window) : max_len);
+  float* part = nullptr;
+  if (splits > 1) {
+    const size_t need = decode_attention_part_floats(b, n_heads, head_dim, splits);
+    if (need > kStaticPartFloats)
+      return set_err(SR_ERR_INVALID_ARG,
+                     "sr_k_decode_attention_static: %zu scratch floats needed (b=%d, heads=%d, head_dim=%d, %d "
+                     "splits of %d positions) but the static scratch holds %zu",
+                     need, b, n_heads, head_dim, splits, SPLIT, kStaticPartFloats);
+    SR_TRY(static_part_ptr(&part));
+  }
+  return launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
+                                 head_dim, window, out, part, splits, static_cast<cudaStream_t>(stream));
+}
