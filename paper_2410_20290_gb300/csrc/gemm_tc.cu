@@ -374,16 +374,18 @@ int g_num_sms = 0;
 int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
 int* g_err = nullptr;
 
-// Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost, the cost
-// growing with BN (MMA and W-tile bytes) plus a fixed part (the A tile and the pipeline fill).
-int pick_bn(int M, int N) {
+// Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost.  The per-tile
+// cost has a part proportional to BN * K (MMA work and W-tile bytes) and a fixed part (A-tile
+// traffic, pipeline fill, epilogue) that a sweep of the decode and scoring shapes on GB300 puts
+// at about the cost of 430 columns of a K = 4096 tile.
+int pick_bn(int M, int N, int K) {
   if (g_bn_override == 64 || g_bn_override == 128 || g_bn_override == 256) return g_bn_override;
   int best = 256;
-  long long best_cost = -1;
+  double best_cost = -1;
   for (int bn : {256, 128, 64}) {
     const long long tiles = (long long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
     const long long waves = (tiles + g_num_sms - 1) / g_num_sms;
-    const long long cost = waves * (bn + 64);
+    const double cost = (double)waves * (bn * (K / 4096.0) + 430.0);
     if (best_cost < 0 || cost < best_cost) best_cost = cost, best = bn;
   }
   return best;
@@ -445,7 +447,7 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     if (const char* e = getenv("SR_GEMM_BN")) g_bn_override = atoi(e);
   }
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
-  const int bn = pick_bn(M, N);
+  const int bn = pick_bn(M, N, K);
   CUtensorMap ta, tb;
   SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
   SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn));

@@ -99,11 +99,11 @@ T16 = {si.DT_BF16: torch.bfloat16, si.DT_F16: torch.float16}
 
 
 @pytest.mark.parametrize("dt", [si.DT_F16, si.DT_BF16])
-# shapes cover all three N-tile widths the launcher picks (64: small tile counts, 128: e.g. 1024 x 6144,
+# shapes cover all three N-tile widths the launcher picks (64: small tile counts, 128: e.g. 308 x 6144,
 # 256: e.g. 1024 x 4096) and ragged M, N and K tails
 @pytest.mark.parametrize("M,N,K", [(1, 256, 64), (7, 512, 128), (130, 2304, 768), (300, 288, 1000), (257, 96, 520),
                                    (1024, 4096, 4096), (1, 32000, 768), (2048, 512, 64), (1024, 6144, 520),
-                                   (308, 28672, 256)])
+                                   (308, 28672, 256), (308, 6144, 512)])
 def test_gemm_tc_fp32_out(sr, dt, M, N, K):
     g = torch.Generator().manual_seed(M * 7 + N + K)
     A = torch.randn(M, K, generator=g).to(T16[dt])
@@ -121,7 +121,7 @@ def test_gemm_tc_fp32_out(sr, dt, M, N, K):
 
 @pytest.mark.parametrize("dt", [si.DT_F16, si.DT_BF16])
 @pytest.mark.parametrize("epi", [2, 3, 4, 5])
-@pytest.mark.parametrize("M,N,K", [(5, 256, 64), (200, 1024, 512), (129, 512, 4096), (1024, 6144, 128),
+@pytest.mark.parametrize("M,N,K", [(5, 256, 64), (200, 1024, 512), (129, 512, 4096), (308, 6144, 512),
                                    (1024, 4096, 64)])
 def test_gemm_tc_epilogues(sr, dt, epi, M, N, K):
     g = torch.Generator().manual_seed(epi * 1000 + M)
