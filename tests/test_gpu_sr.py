@@ -216,9 +216,22 @@ def _teacher_forced(sr, w, seed, prompt, n_steps):
 
 
 def test_gpt2_shaped_teacher_forced(sr):
-    """GPT-2-small widths (LayerNorm, GELU, learned positions, bf16), 2 layers, 16 candidates."""
-    w = si.shrink(si.WORKLOADS["gpt2"], 2, N=16, max_new=24, taus=(12,))
+    """GPT-2-small shape at full depth (12 layers, LayerNorm, GELU, learned positions, bf16 weights), 16
+    candidates, the workload's 128-token prompt."""
+    w = si.WORKLOADS["gpt2"].replace(N=16, max_new=24, taus=(12,))
     worst = _teacher_forced(sr, w, 0, w.prompt(0), 20)
+    assert worst <= LOGIT_TOL
+
+
+@pytest.mark.parametrize("window", [4096, 24])
+def test_mistral_rm2b_shaped_teacher_forced(sr, window):
+    """Mistral-7B widths (GQA 32/8, vocab 32000) with the 2B-shaped reward model (MHA, head_dim 256, GeGLU
+    16384), 2 layers each, 8 candidates.  The workload's 4096-position window never binds at these lengths, so
+    a 24-position window also runs, which the decode and prefill attention must apply."""
+    base = si.WORKLOADS["mistral7b_rm2b"]
+    w = si.shrink(base, 2, N=8, max_new=14, taus=(7,), prompt_len=21, sched_kind=si.SCHED_FIXED, pool_bytes=0)
+    w = w.replace(gen=w.gen.replace(window=window), rm=w.rm.replace(window=window))
+    worst = _teacher_forced(sr, w, 0, w.prompt(0), 12)
     assert worst <= LOGIT_TOL
 
 
