@@ -255,10 +255,14 @@ sr_status sr_k_gemm(int dtype, const void* A, const void* W, void* C, int M, int
  * and query head j, out[s][j] = softmax_t(q[s][j] . K_t / sqrt(dh)) V_t over
  * positions t in [max(0, len[s] - window), len[s]) read from the pool pages
  * page_table[orig_ids[s]][t / 16].  pool layout [page][2 (K,V)][n_kv][16][dh]
- * of `dtype` (pool points at this layer's page 0); q, out [b][n_heads][dh] `dtype`. */
+ * of `dtype` (pool points at this layer's page 0); q, out [b][n_heads][dh] `dtype`.
+ * shared_pos (a multiple of 16, < every len; 0 = none): positions [0, shared_pos)
+ * are in the same pages for every candidate (the shared prompt, Section 4.2's batch
+ * of N responses to one prompt) and are read once per 64 candidates by a
+ * tensor-core prefix pass (16-bit types only). */
 sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, const int32_t* page_table, int pt_stride,
                                 const int32_t* orig_ids, const int32_t* lens, int b, int n_heads, int n_kv_heads,
-                                int head_dim, int window, void* out, void* stream);
+                                int head_dim, int window, int shared_pos, void* out, void* stream);
 
 /* sr_k_decode_attention_static -- the same decode attention for callers that cannot allocate
  * device memory when they call (a server that has reserved all GPU memory up front, an

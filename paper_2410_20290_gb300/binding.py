@@ -89,7 +89,7 @@ _SIG = {
     "sr_k_sample": [_P, ctypes.c_longlong, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P],
     "sr_k_rcut": [_P, _I, _F, _I, _P, _P, _P],
     "sr_k_gemm": [_I, _P, _P, _P, _I, _I, _I, _I, _P],
-    "sr_k_decode_attention": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P, _P],
+    "sr_k_decode_attention": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P],
     "sr_k_decode_attention_static": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P],
     "sr_k_prefill_attention": [_I, _P, _P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _I, _P, _P],
 }
@@ -268,9 +268,9 @@ def sr_k_gemm(dtype, A, W, C, M, N, K, epilogue, stream=None):
 
 
 def sr_k_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads, head_dim,
-                          window, out, stream=None):
+                          window, out, stream=None, shared_pos=0):
     _check(LIB.sr_k_decode_attention(dtype, _ptr(q), _ptr(pool), _ptr(page_table), pt_stride, _ptr(orig_ids),
-                                     _ptr(lens), b, n_heads, n_kv_heads, head_dim, window, _ptr(out),
+                                     _ptr(lens), b, n_heads, n_kv_heads, head_dim, window, shared_pos, _ptr(out),
                                      _stream(stream)))
 
 

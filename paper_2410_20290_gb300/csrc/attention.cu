@@ -135,20 +135,23 @@ __global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, co
   }
 }
 
+// Merges the partial (O, m, l) of each split; with a shared-prefix pass, partial slot 0 holds the
+// prefix and the position splits start at slot 1 (sbase = 1, suffix positions from t_min).
 template <typename T, int DH>
 __global__ void k_decode_combine(const float* __restrict__ part, const int* __restrict__ lens, int Hq, int window,
-                                 int max_splits, T* __restrict__ out) {
+                                 int max_splits, int t_min, int sbase, T* __restrict__ out) {
   const int hq = blockIdx.x, s = blockIdx.y, d = threadIdx.x;
   const int L = lens[s];
-  const int t_lo = window > 0 ? max(0, L - window) : 0;
-  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
-  if (nsplit <= 1) return;  // written directly by k_decode_attn
+  const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
+  const int total = sbase + (L - t_lo + SPLIT - 1) / SPLIT;
+  if (total <= 1) return;  // written directly by the attention kernel
   const float* pp = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
   float M = -INFINITY;
-  for (int j = 0; j < nsplit; ++j) M = fmaxf(M, pp[j * (DH + 2) + DH]);
+  for (int j = 0; j < total; ++j) M = fmaxf(M, pp[j * (DH + 2) + DH]);
   float Lsum = 0.f, O = 0.f;
-  for (int j = 0; j < nsplit; ++j) {
-    const float w = exp2f(pp[j * (DH + 2) + DH] - M);
+  for (int j = 0; j < total; ++j) {
+    const float mj = pp[j * (DH + 2) + DH];
+    const float w = (mj == -INFINITY) ? 0.f : exp2f(mj - M);
     Lsum += pp[j * (DH + 2) + DH + 1] * w;
     O += pp[j * (DH + 2) + d] * w;
   }
@@ -236,8 +239,8 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
                                                         const int* __restrict__ pt, int pt_stride,
                                                         const int* __restrict__ slot_ids,
                                                         const int* __restrict__ lens, int Hkv, float scale_log2,
-                                                        int window, int max_splits, T* __restrict__ out,
-                                                        float* __restrict__ part) {
+                                                        int window, int t_min, int sbase, int max_splits,
+                                                        T* __restrict__ out, float* __restrict__ part) {
   static_assert(G >= 1 && G <= 8 && DH % 16 == 0, "shape");
   constexpr int LDS = DH + 8;                  // padded smem row (elements): conflict-free ldmatrix
   constexpr int BLK = PAGE * LDS;              // one K or V page block in smem
@@ -253,7 +256,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
   const int h = blockIdx.x, s = blockIdx.y, split = blockIdx.z;
   const int Hq = Hkv * G;
   const int L = lens[s];
-  const int t_lo = window > 0 ? max(0, L - window) : 0;
+  const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
   const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
   if (split >= nsplit) return;
   const int t_begin = t_lo + split * SPLIT, t_end = min(L, t_begin + SPLIT);
@@ -394,10 +397,10 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       O += so[((size_t)w * DH + d) * 8 + j] * wt;
     }
     const int hq = h * G + j;
-    if (nsplit == 1) {
+    if (nsplit == 1 && sbase == 0) {
       out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
     } else {
-      float* pp = part + (((size_t)s * Hq + hq) * max_splits + split) * (DH + 2);
+      float* pp = part + (((size_t)s * Hq + hq) * max_splits + sbase + split) * (DH + 2);
       pp[d] = O;
       if (d == 0) pp[DH] = M, pp[DH + 1] = Lsum;
     }
@@ -572,6 +575,157 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
   }
 }
 
+
+// Shared-prompt prefix of decode attention.  Positions [0, S) sit in pages every live candidate shares
+// (the prompt's full pages), so instead of each candidate re-reading them, one CTA takes 64 candidates'
+// queries for one query head and runs flash attention over the prefix keys with mma.sync: each prefix
+// K/V block is loaded once per 64 candidates.  The result is written unnormalised as partial slot 0
+// (O, m, l in the decode kernels' log2-scaled convention) for k_decode_combine to merge with the suffix
+// partials.  No causal mask is needed (every prefix position precedes the query); a window masks per row.
+template <typename T, int DH>
+__global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, const T* __restrict__ pool,
+                                                     const int* __restrict__ pt, int pt_stride,
+                                                     const int* __restrict__ slot_ids,
+                                                     const int* __restrict__ lens, int n, int S, int Hq, int Hkv,
+                                                     float scale_log2, int window, int max_splits,
+                                                     float* __restrict__ part) {
+  constexpr int LD = DH + 8;
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  T* sQ = reinterpret_cast<T*>(smem_raw);
+  T* sK = sQ + BQ * LD;
+  T* sV = sK + BKV * LD;
+  const int s0 = blockIdx.x * BQ, hq = blockIdx.y, hk = hq / (Hq / Hkv);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
+  const int* prow = pt + (size_t)slot_ids[0] * pt_stride;   // the prompt pages, identical in every row
+  const size_t page_elems = (size_t)2 * Hkv * PAGE * DH;
+  const size_t v_off = (size_t)Hkv * PAGE * DH;
+
+  for (int c = tid; c < BQ * (DH / 8); c += 128) {
+    const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+    const bool ok = s0 + row < n;
+    const T* src = ok ? q + ((size_t)(s0 + row) * Hq + hq) * DH + col : q;
+    cp_async16(sQ + row * LD + col, src, ok);
+  }
+  float o[DH / 8][4];
+#pragma unroll
+  for (int i = 0; i < DH / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  int qpos[2];
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int row = s0 + warp * 16 + g + 8 * r;
+    qpos[r] = row < n ? lens[row] - 1 : 0;
+  }
+  const int nb = (S + BKV - 1) / BKV;
+  for (int kb = 0; kb < nb; ++kb) {
+    const int kbase = kb * BKV, kcount = min(BKV, S - kbase);
+    __syncthreads();
+    for (int c = tid; c < BKV * (DH / 8); c += 128) {
+      const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+      const bool ok = row < kcount;
+      const int key = kbase + row;
+      const T* src = pool;
+      if (ok) src = pool + (size_t)prow[key / PAGE] * page_elems + ((size_t)hk * PAGE + key % PAGE) * DH + col;
+      cp_async16(sK + row * LD + col, src, ok);
+      cp_async16(sV + row * LD + col, ok ? src + v_off : pool, ok);
+    }
+    cp_async_wait_all();
+    __syncthreads();
+    float sc[BKV / 8][4];
+#pragma unroll
+    for (int i = 0; i < BKV / 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < DH / 16; ++kk) {
+      uint32_t a0, a1, a2, a3;
+      ldm_x4(smem_addr(sQ + (warp * 16 + (lane & 15)) * LD + kk * 16 + (lane >> 4) * 8), a0, a1, a2, a3);
+#pragma unroll
+      for (int np = 0; np < BKV / 16; ++np) {
+        uint32_t b0, b1, b2, b3;
+        ldm_x4(smem_addr(sK + (np * 16 + (lane & 7) + ((lane >> 4) << 3)) * LD + kk * 16 + ((lane >> 3) & 1) * 8), b0,
+               b1, b2, b3);
+        mma16816<T>(sc[2 * np], a0, a1, a2, a3, b0, b1);
+        mma16816<T>(sc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+    float bmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int nt = 0; nt < BKV / 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int kidx = nt * 8 + 2 * t4 + (e & 1);
+        const int r = e >> 1;
+        bool ok = kidx < kcount;
+        if (window > 0) ok = ok && kbase + kidx > qpos[r] - window;
+        const float x = ok ? sc[nt][e] * scale_log2 : -INFINITY;
+        sc[nt][e] = x;
+        bmax[r] = fmaxf(bmax[r], x);
+      }
+    }
+    float corr[2], base[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      bmax[r] = fmaxf(bmax[r], __shfl_xor_sync(0xffffffffu, bmax[r], 1));
+      bmax[r] = fmaxf(bmax[r], __shfl_xor_sync(0xffffffffu, bmax[r], 2));
+      const float mn = fmaxf(mrow[r], bmax[r]);
+      base[r] = (mn == -INFINITY) ? 0.f : mn;
+      corr[r] = exp2f(mrow[r] - base[r]);
+      mrow[r] = mn;
+    }
+    float psum[2] = {0.f, 0.f};
+#pragma unroll
+    for (int nt = 0; nt < BKV / 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float p = exp2f(sc[nt][e] - base[e >> 1]);
+        sc[nt][e] = p;
+        psum[e >> 1] += p;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) lrow[r] = lrow[r] * corr[r] + psum[r];
+#pragma unroll
+    for (int i = 0; i < DH / 8; ++i) {
+      o[i][0] *= corr[0], o[i][1] *= corr[0];
+      o[i][2] *= corr[1], o[i][3] *= corr[1];
+    }
+#pragma unroll
+    for (int kk = 0; kk < BKV / 16; ++kk) {
+      uint32_t ah[4], al[4];
+      split16<T>(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+      split16<T>(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+      split16<T>(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+      split16<T>(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
+#pragma unroll
+      for (int dp = 0; dp < DH / 16; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LD + dp * 16 + (lane >> 4) * 8), b0,
+                 b1, b2, b3);
+        mma16816<T>(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
+        mma16816<T>(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+        mma16816<T>(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
+        mma16816<T>(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+    lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+  }
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int row = s0 + warp * 16 + g + 8 * r;
+    if (row >= n) continue;
+    float* pp = part + ((size_t)row * Hq + hq) * max_splits * (DH + 2);   // partial slot 0
+#pragma unroll
+    for (int nt = 0; nt < DH / 8; ++nt) {
+      pp[nt * 8 + 2 * t4] = o[nt][2 * r];
+      pp[nt * 8 + 2 * t4 + 1] = o[nt][2 * r + 1];
+    }
+    if (t4 == 0) pp[DH] = mrow[r], pp[DH + 1] = lrow[r];
+  }
+}
+
 // fp32 models: straightforward prefill attention, one block per (query row, head); scores of the
 // row's visible keys live in shared memory.
 __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __restrict__ k,
@@ -626,7 +780,23 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
 template <typename T, int DH, int G>
 sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
                            const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
-                           cudaStream_t st) {
+                           int shared_pos, cudaStream_t st) {
+  // with a shared prefix: slot 0 of the partials is the prefix pass, position splits follow
+  const int sbase = shared_pos > 0 ? 1 : 0;
+  const int t_min = shared_pos;
+  if (sbase) {
+    if (!part) return set_err(SR_ERR_INVALID_ARG, "decode attention: partial buffer missing for the prefix pass");
+    const size_t psmem = (size_t)(BQ + 2 * BKV) * (DH + 8) * sizeof(T);
+    static bool pattr = false;
+    if (!pattr) {
+      SR_CUDA(cudaFuncSetAttribute(k_prefix_attn<T, DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem));
+      pattr = true;
+    }
+    k_prefix_attn<T, DH><<<dim3((b + BQ - 1) / BQ, Hkv * G), 128, psmem, st>>>(
+        (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, b, shared_pos, Hkv * G, Hkv,
+        1.4426950408889634f / sqrtf((float)DH), window, max_splits, part);
+    SR_LAUNCH();
+  }
   constexpr int LDS = DH + 8;
   const size_t smem = std::max<size_t>((size_t)4 * (2 * 2 * PAGE * LDS + 2 * 8 * PAGE) * sizeof(T),
                                        (size_t)(64 + 4 * DH * 8) * sizeof(float));
@@ -636,12 +806,13 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
-  dim3 grid(Hkv, b, max_splits);
+  dim3 grid(Hkv, b, max_splits - sbase);
   k_decode_attn_tc<T, DH, G><<<grid, 128, smem, st>>>((const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
-                                                       scale_log2, window, max_splits, (T*)out, part);
+                                                       scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
   SR_LAUNCH();
   if (max_splits > 1) {
-    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, (T*)out);
+    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, t_min, sbase,
+                                                             (T*)out);
     SR_LAUNCH();
   }
   return SR_OK;
@@ -657,7 +828,8 @@ sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_s
                                                  scale_log2, window, max_splits, (T*)out, part);
   SR_LAUNCH();
   if (max_splits > 1) {
-    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, (T*)out);
+    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, 0, 0,
+                                                             (T*)out);
     SR_LAUNCH();
   }
   return SR_OK;
@@ -685,13 +857,18 @@ sr_status prefill_t(const void* q, const void* k, const void* v, const void* kpr
 }  // namespace
 
 int decode_attention_max_splits(int max_len) { return max_len <= 0 ? 1 : (max_len + SPLIT - 1) / SPLIT; }
+int decode_attention_slots(int max_len, int window, int shared_pos) {
+  const int lo = shared_pos > 0 ? shared_pos : 0;
+  const int span = window > 0 ? std::min(max_len - lo, window) : max_len - lo;
+  return (shared_pos > 0 ? 1 : 0) + decode_attention_max_splits(span);
+}
 size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits) {
   return (size_t)b * Hq * max_splits * (dh + 2);
 }
 
 sr_status launch_decode_attention(int et, const void* q, const void* pool_layer, const int* pt, int pt_stride,
                                   const int* ids, const int* lens, int b, int Hq, int Hkv, int dh, int window,
-                                  void* out, float* part, int max_splits, cudaStream_t st) {
+                                  void* out, float* part, int max_splits, cudaStream_t st, int shared_pos) {
   if (b == 0) return SR_OK;
   const int G = Hq / Hkv;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "decode attention: n_heads %% n_kv_heads != 0");
@@ -703,13 +880,14 @@ sr_status launch_decode_attention(int et, const void* q, const void* pool_layer,
 #define SR_DECT(T, D, GG)                                                                                          \
   if (dh == D && G == GG)                                                                                            \
     return decode_attn_tc_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
-                                      st);
+                                      shared_pos, st);
   if (et == SR_DT_F16) {
     SR_DECT(f16, 128, 4) SR_DECT(f16, 128, 1) SR_DECT(f16, 128, 2) SR_DECT(f16, 128, 8)
     SR_DECT(f16, 64, 1) SR_DECT(f16, 64, 4) SR_DECT(f16, 32, 1)
   } else if (et == SR_DT_BF16) {
     SR_DECT(bf16, 128, 4) SR_DECT(bf16, 128, 1) SR_DECT(bf16, 64, 1)
   } else {
+    if (shared_pos > 0) return set_err(SR_ERR_UNSUPPORTED, "decode attention: shared-prefix pass needs 16-bit KV");
     SR_DEC(float, 32, 1) SR_DEC(float, 32, 2) SR_DEC(float, 32, 4) SR_DEC(float, 64, 1) SR_DEC(float, 128, 1)
     SR_DEC(float, 8, 1) SR_DEC(float, 8, 2) SR_DEC(float, 8, 4)
   }

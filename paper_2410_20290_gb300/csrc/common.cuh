@@ -162,10 +162,15 @@ sr_status launch_sample(const float* logits, long long ld, int b, int V, const i
                         int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st);
 
 // attention.cu
+// shared_pos > 0: positions [0, shared_pos) sit in pages shared by every row's page table (the prompt);
+// a tensor-core prefix pass reads them once per 64 rows and `part` must hold
+// decode_attention_slots(max_len, window, shared_pos) partial slots per (row, head).
 sr_status launch_decode_attention(int dtype, const void* q, const void* pool_layer, const int* page_table,
                                   int pt_stride, const int* slot_ids, const int* lens, int b, int Hq, int Hkv, int dh,
-                                  int window, void* out, float* part, int max_splits, cudaStream_t st);
+                                  int window, void* out, float* part, int max_splits, cudaStream_t st,
+                                  int shared_pos = 0);
 int decode_attention_max_splits(int max_len);
+int decode_attention_slots(int max_len, int window, int shared_pos);
 size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits);
 sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* k_pre,
                                        const float* v_pre, int n_pre, const int* seq_off, int n_seq, int rows,

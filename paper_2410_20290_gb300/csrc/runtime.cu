@@ -647,7 +647,10 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
   }
   const int max_len = b.P + b.g;
   const int eff_len = d.window > 0 ? std::min(max_len, d.window) : max_len;
-  const int splits = decode_attention_max_splits(eff_len);
+  // the prompt's full pages are shared by every candidate: a tensor-core prefix pass reads them once per 64
+  // candidates (16-bit KV only)
+  const int shared_pos = (m.et == SR_DT_F16 && b.n_sh > 0) ? PAGE * b.n_sh : 0;
+  const int splits = decode_attention_slots(max_len, d.window, shared_pos);
   if (splits > 1) SR_TRY(grow(w.part, w.c_part, decode_attention_part_floats(n, Hq, dh, splits)));
   // algorithmic work of one decode-attention launch: the shared prompt KV once, each candidate's own KV,
   // q in and the output out
@@ -675,7 +678,7 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
     {
       Scope sc(pf, SR_KC_ATTN_DECODE, st, attn_flops, attn_bytes);
       SR_TRY(launch_decode_attention(m.et, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
-                                     d.window, w.att, w.part, splits, st));
+                                     d.window, w.att, w.part, splits, st, shared_pos));
     }
     SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, st, pf, SR_KC_GEMM_DECODE));
     {
@@ -1231,7 +1234,7 @@ sr_status sr_k_gemm(int dtype, const void* A, const void* W, void* C, int M, int
 
 sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, const int32_t* page_table, int pt_stride,
                                 const int32_t* orig_ids, const int32_t* lens, int b, int n_heads, int n_kv_heads,
-                                int head_dim, int window, void* out, void* stream) {
+                                int head_dim, int window, int shared_pos, void* out, void* stream) {
   if (!q || !pool || !page_table || !orig_ids || !lens || !out) return set_err(SR_ERR_INVALID_ARG, "null argument");
   if (b < 0 || n_kv_heads < 1 || n_heads < 1 || head_dim < 1) return set_err(SR_ERR_INVALID_ARG, "bad shape");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1240,12 +1243,15 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
   if (b) SR_CUDA(cudaMemcpy(h.data(), lens, b * sizeof(int), cudaMemcpyDeviceToHost));
   int mx = 1;
   for (int x : h) mx = std::max(mx, x);
-  const int splits = decode_attention_max_splits(window > 0 ? std::min(mx, window) : mx);
+  if (shared_pos < 0 || shared_pos % PAGE) return set_err(SR_ERR_INVALID_ARG, "shared_pos must be a multiple of 16");
+  for (int x : h)
+    if (x <= shared_pos) return set_err(SR_ERR_INVALID_ARG, "every length must exceed shared_pos");
+  const int splits = decode_attention_slots(mx, window, shared_pos);
   float* part = nullptr;
   if (splits > 1) SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&part),
                                           decode_attention_part_floats(b, n_heads, head_dim, splits) * sizeof(float), st));
   sr_status s = launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
-                                        head_dim, window, out, part, splits, st);
+                                        head_dim, window, out, part, splits, st, shared_pos);
   if (part) cudaFreeAsync(part, st);
   return s;
 }

@@ -1,7 +1,7 @@
 """Time one libsr kernel on synthetic inputs through the C ABI (CUDA events, after warm-up).
 
   python -m paper_2410_20290_gb300.microbench gemm M N K [epilogue]
-  python -m paper_2410_20290_gb300.microbench decode_attn b Hq Hkv dh len
+  python -m paper_2410_20290_gb300.microbench decode_attn b Hq Hkv dh len [shared_positions]
   python -m paper_2410_20290_gb300.microbench prefill_attn n_seq tau n_pre Hq Hkv dh
   python -m paper_2410_20290_gb300.microbench sample b V
 
@@ -49,19 +49,22 @@ def gemm(M, N, K, epi=0, iters=20):
     return dict(kernel="gemm", M=M, N=N, K=K, epi=epi, ms=ms, tflops=fl / ms / 1e9, gbs=by / ms / 1e6)
 
 
-def decode_attn(b, Hq, Hkv, dh, L, iters=20):
+def decode_attn(b, Hq, Hkv, dh, L, shared=0, iters=20):
+    """shared > 0: the first `shared` positions sit in pages common to every candidate (the prompt)."""
     pages = (L + 15) // 16
-    pool = torch.randn(b * pages + 1, 2, Hkv, 16, dh, device="cuda").to(torch.float16)
-    pt = torch.randperm(b * pages, device="cuda").to(torch.int32).reshape(b, pages)
+    sp = shared // 16
+    pool = torch.randn(b * (pages - sp) + sp + 1, 2, Hkv, 16, dh, device="cuda").to(torch.float16)
+    own = torch.randperm(b * (pages - sp), device="cuda").to(torch.int32).reshape(b, pages - sp) + sp
+    pt = torch.cat([torch.arange(sp, device="cuda", dtype=torch.int32).expand(b, sp), own], 1).contiguous()
     ids = torch.arange(b, device="cuda", dtype=torch.int32)
     lens = torch.full((b,), L, device="cuda", dtype=torch.int32)
     q = torch.randn(b, Hq, dh, device="cuda").to(torch.float16)
     out = torch.zeros_like(q)
     s = torch.cuda.current_stream().cuda_stream
-    ms = _time(lambda: sr.sr_k_decode_attention(DT_F16, q, pool, pt, pages, ids, lens, b, Hq, Hkv, dh, 0, out, s),
-               iters)
-    by = b * L * Hkv * dh * 2 * 2 + 2 * q.numel() * 2
-    return dict(kernel="decode_attn", b=b, Hq=Hq, Hkv=Hkv, dh=dh, len=L, ms=ms, gbs=by / ms / 1e6)
+    ms = _time(lambda: sr.sr_k_decode_attention(DT_F16, q, pool, pt, pages, ids, lens, b, Hq, Hkv, dh, 0, out, s,
+                                                shared_pos=shared), iters)
+    by = (b * (L - shared) + shared) * Hkv * dh * 2 * 2 + 2 * q.numel() * 2    # shared positions counted once
+    return dict(kernel="decode_attn", b=b, Hq=Hq, Hkv=Hkv, dh=dh, len=L, shared=shared, ms=ms, gbs=by / ms / 1e6)
 
 
 def prefill_attn(n_seq, tau, n_pre, Hq, Hkv, dh, iters=10):

@@ -157,16 +157,22 @@ def _round16(x, dt=si.DT_F16):
     return torch.from_numpy(x).to(T16[dt]).float().numpy()
 
 
-@pytest.mark.parametrize("dt,Hq,Hkv,dh,window,lens", [
-    (si.DT_F16, 32, 8, 128, 0, [1, 15, 16, 17, 300, 511, 512, 513, 1100, 2000]),
-    (si.DT_F16, 12, 12, 64, 0, [5, 129, 700]),
-    (si.DT_F16, 32, 8, 128, 100, [50, 100, 101, 900]),
-    (si.DT_F16, 16, 2, 128, 0, [33, 64, 600]),
-    (si.DT_F16, 4, 4, 32, 0, [1, 16, 33, 80]),
-    (si.DT_BF16, 32, 8, 128, 0, [7, 300, 1300]),
-    (si.DT_F32, 4, 4, 32, 0, [1, 16, 33, 80]),
+@pytest.mark.parametrize("dt,Hq,Hkv,dh,window,lens,shared", [
+    (si.DT_F16, 32, 8, 128, 0, [1, 15, 16, 17, 300, 511, 512, 513, 1100, 2000], 0),
+    (si.DT_F16, 12, 12, 64, 0, [5, 129, 700], 0),
+    (si.DT_F16, 32, 8, 128, 100, [50, 100, 101, 900], 0),
+    (si.DT_F16, 16, 2, 128, 0, [33, 64, 600], 0),
+    (si.DT_F16, 4, 4, 32, 0, [1, 16, 33, 80], 0),
+    (si.DT_BF16, 32, 8, 128, 0, [7, 300, 1300], 0),
+    (si.DT_F32, 4, 4, 32, 0, [1, 16, 33, 80], 0),
+    # shared prompt pages: the tensor-core prefix pass plus the suffix splits
+    (si.DT_F16, 32, 8, 128, 0, [289, 290, 300, 511, 800, 805, 1300] * 10, 288),
+    (si.DT_F16, 12, 12, 64, 0, [129, 130, 700], 128),
+    (si.DT_F16, 32, 8, 128, 40, [300, 301, 305], 256),
+    (si.DT_F16, 32, 8, 128, 0, [17, 18, 600], 16),
+    (si.DT_BF16, 32, 8, 128, 0, [300, 900], 272),
 ])
-def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens):
+def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens, shared):
     rng = np.random.default_rng(dh + len(lens))
     b = len(lens)
     max_pages = max(lens) // 16 + 1
@@ -177,11 +183,12 @@ def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens):
         pool, q = _round16(pool, dt), _round16(q, dt)
     perm = rng.permutation(n_pages).astype(np.int32)
     ids = rng.permutation(b).astype(np.int32)                       # slot s serves candidate ids[s]
-    pt = perm[: b * max_pages].reshape(b, max_pages)                # page table indexed by candidate id
+    pt = perm[: b * max_pages].reshape(b, max_pages).copy()         # page table indexed by candidate id
+    pt[:, : shared // 16] = pt[0, : shared // 16]                   # the shared prompt pages
     tdt = T16.get(dt, torch.float32)
     out = torch.zeros(b, Hq, dh, dtype=tdt, device="cuda")
     sr.sr_k_decode_attention(dt, dev(q, tdt), dev(pool, tdt), dev(pt), max_pages, dev(ids),
-                             dev(np.array(lens, np.int32)), b, Hq, Hkv, dh, window, out)
+                             dev(np.array(lens, np.int32)), b, Hq, Hkv, dh, window, out, shared_pos=shared)
     got = out.float().cpu().numpy()
     for s in range(b):
         L = lens[s]

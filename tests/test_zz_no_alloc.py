@@ -42,7 +42,7 @@ def _run(sr, c, static, window=0):
     if static:
         sr.sr_k_decode_attention_static(*args, int(c["lens"].max()), out)
     else:
-        sr.sr_k_decode_attention(*args, out)
+        sr.sr_k_decode_attention(*args, out)    # no shared prefix: the same kernels as the static entry point
     torch.cuda.synchronize()
     return out.float().cpu()
 
