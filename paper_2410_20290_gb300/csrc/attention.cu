@@ -336,8 +336,9 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       m[j] = mn;
       // P[head][position] as hi + lo 16-bit values
       const int hc = 2 * t4 + j;
-      uint32_t hi, lo;
-      split16<T>(p0, p1, hi, lo);
+      uint32_t hi, lo = 0u;
+      if constexpr (std::is_same<T, bf16>::value) split16<T>(p0, p1, hi, lo);
+      else hi = pack2<T>(p0, p1);
       sPh[hc * PAGE + g] = (uint16_t)(hi & 0xFFFFu);
       sPh[hc * PAGE + g + 8] = (uint16_t)(hi >> 16);
       sPl[hc * PAGE + g] = (uint16_t)(lo & 0xFFFFu);
@@ -361,7 +362,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       const int mi = lane >> 3, r = lane & 7;
       ldm_x4_t(smem_addr(sV + (r + ((mi >> 1) << 3)) * LDS + mt * 16 + (mi & 1) * 8), a0, a1, a2, a3);
       mma16816<T>(o[mt], a0, a1, a2, a3, bh0, bh1);
-      mma16816<T>(o[mt], a0, a1, a2, a3, bl0, bl1);
+      if constexpr (std::is_same<T, bf16>::value) mma16816<T>(o[mt], a0, a1, a2, a3, bl0, bl1);
     }
     __syncwarp();
     if (i + 2 < my_pages) issue(i + 2, stage);
@@ -403,6 +404,40 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       float* pp = part + (((size_t)s * Hq + hq) * max_splits + sbase + split) * (DH + 2);
       pp[d] = O;
       if (d == 0) pp[DH] = M, pp[DH + 1] = Lsum;
+    }
+  }
+}
+
+// O[16 x 16*NDP] += P[16 x 64] V[64 x 16*NDP] for one warp: P comes from the S accumulators (C layout of
+// m16n8k16), V rows are read transposed from shared memory.  fp16 P is used as is (11-bit significand);
+// bf16 P is split into hi + lo pairs (two MMAs) to keep ~16 significand bits.
+template <typename T, int NDP>
+__device__ __forceinline__ void pv_accumulate(const float (*sc)[4], const T* sV, int ldv, int lane, float (*o)[4]) {
+#pragma unroll
+  for (int kk = 0; kk < 4; ++kk) {
+    uint32_t ah[4], al[4];
+    if constexpr (std::is_same<T, bf16>::value) {
+      split16<T>(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+      split16<T>(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+      split16<T>(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+      split16<T>(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
+    } else {
+      ah[0] = pack2<T>(sc[2 * kk][0], sc[2 * kk][1]);
+      ah[1] = pack2<T>(sc[2 * kk][2], sc[2 * kk][3]);
+      ah[2] = pack2<T>(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      ah[3] = pack2<T>(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+    }
+#pragma unroll
+    for (int dp = 0; dp < NDP; ++dp) {
+      uint32_t b0, b1, b2, b3;
+      ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * ldv + dp * 16 + (lane >> 4) * 8), b0,
+               b1, b2, b3);
+      mma16816<T>(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
+      mma16816<T>(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+      if constexpr (std::is_same<T, bf16>::value) {
+        mma16816<T>(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
+        mma16816<T>(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
+      }
     }
   }
 }
@@ -536,26 +571,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
       o[i][0] *= corr[0], o[i][1] *= corr[0];
       o[i][2] *= corr[1], o[i][3] *= corr[1];
     }
-    // O += P V, with P carried as a bf16 hi + lo pair (P = hi + lo to ~16 mantissa bits) so the
-    // probabilities are not the coarsest operand in the product
-#pragma unroll
-    for (int kk = 0; kk < BKV / 16; ++kk) {
-      uint32_t ah[4], al[4];
-      split16<T>(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
-      split16<T>(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
-      split16<T>(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
-      split16<T>(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
-#pragma unroll
-      for (int dp = 0; dp < DV / 16; ++dp) {
-        uint32_t b0, b1, b2, b3;
-        ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LDV + dp * 16 + (lane >> 4) * 8), b0,
-                 b1, b2, b3);
-        mma16816<T>(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
-        mma16816<T>(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
-        mma16816<T>(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
-        mma16816<T>(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
-      }
-    }
+    // O += P V (bf16 carries P as a hi + lo pair so the probabilities are not the coarsest operand)
+    pv_accumulate<T, DV / 16>(sc, sV, LDV, lane, o);
   }
   // finish: full row sums across the quad, normalise, store
 #pragma unroll
@@ -577,35 +594,59 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
 
 
 // Shared-prompt prefix of decode attention.  Positions [0, S) sit in pages every live candidate shares
-// (the prompt's full pages), so instead of each candidate re-reading them, one CTA takes 64 candidates'
-// queries for one query head and runs flash attention over the prefix keys with mma.sync: each prefix
-// K/V block is loaded once per 64 candidates.  The result is written unnormalised as partial slot 0
-// (O, m, l in the decode kernels' log2-scaled convention) for k_decode_combine to merge with the suffix
-// partials.  No causal mask is needed (every prefix position precedes the query); a window masks per row.
-template <typename T, int DH>
+// (the prompt's full pages), so instead of each candidate re-reading them, one CTA takes the queries of
+// several candidates for up to 4 query heads of one kv head (64 query rows, one warp per 16 rows) and runs
+// flash attention over the prefix keys with mma.sync; each 64-position K/V block is loaded once per CTA
+// through a 2-stage cp.async pipeline.  The result is written unnormalised as partial slot 0 (O, m, l in
+// the decode kernels' log2-scaled convention) for k_decode_combine to merge with the suffix partials.
+// No causal mask is needed (every prefix position precedes the query); a window masks per row.
+template <typename T, int DH, int G>
 __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, const T* __restrict__ pool,
                                                      const int* __restrict__ pt, int pt_stride,
                                                      const int* __restrict__ slot_ids,
-                                                     const int* __restrict__ lens, int n, int S, int Hq, int Hkv,
+                                                     const int* __restrict__ lens, int n, int S, int Hkv,
                                                      float scale_log2, int window, int max_splits,
                                                      float* __restrict__ part) {
+  constexpr int HPC = G < 4 ? G : 4;       // query heads per CTA
+  constexpr int CPC = 4 / HPC;             // 16-candidate blocks per CTA
   constexpr int LD = DH + 8;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   T* sQ = reinterpret_cast<T*>(smem_raw);
-  T* sK = sQ + BQ * LD;
-  T* sV = sK + BKV * LD;
-  const int s0 = blockIdx.x * BQ, hq = blockIdx.y, hk = hq / (Hq / Hkv);
+  T* sKV = sQ + BQ * LD;                   // [stage][K | V][64][LD]
+  const int Hq = Hkv * G;
+  const int h = blockIdx.y / (G / HPC), hg0 = (blockIdx.y % (G / HPC)) * HPC;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
+  const int wh = warp % HPC, wc = warp / HPC;
+  const int hq = h * G + hg0 + wh;
+  const int s0 = blockIdx.x * 16 * CPC + wc * 16;       // this warp's first candidate row
   const int* prow = pt + (size_t)slot_ids[0] * pt_stride;   // the prompt pages, identical in every row
   const size_t page_elems = (size_t)2 * Hkv * PAGE * DH;
   const size_t v_off = (size_t)Hkv * PAGE * DH;
 
-  for (int c = tid; c < BQ * (DH / 8); c += 128) {
+  // Q rows: warp w's 16 rows are (candidates s0 .. s0 + 15, head hq)
+  for (int c = lane; c < 16 * (DH / 8); c += 32) {
     const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
     const bool ok = s0 + row < n;
     const T* src = ok ? q + ((size_t)(s0 + row) * Hq + hq) * DH + col : q;
-    cp_async16(sQ + row * LD + col, src, ok);
+    cp_async16(sQ + (warp * 16 + row) * LD + col, src, ok);
   }
+  const int nb = (S + BKV - 1) / BKV;
+  auto issue = [&](int kb) {
+    T* dK = sKV + (size_t)(kb & 1) * 2 * BKV * LD;
+    T* dV = dK + BKV * LD;
+    const int kbase = kb * BKV, kcount = min(BKV, S - kbase);
+    for (int c = tid; c < BKV * (DH / 8); c += 128) {
+      const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+      const bool ok = row < kcount;
+      const int key = kbase + row;
+      const T* src = ok ? pool + (size_t)prow[key / PAGE] * page_elems + ((size_t)h * PAGE + key % PAGE) * DH + col
+                        : pool;
+      cp_async16(dK + row * LD + col, src, ok);
+      cp_async16(dV + row * LD + col, ok ? src + v_off : pool, ok);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+
   float o[DH / 8][4];
 #pragma unroll
   for (int i = 0; i < DH / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
@@ -613,24 +654,21 @@ __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, co
   int qpos[2];
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
-    const int row = s0 + warp * 16 + g + 8 * r;
+    const int row = s0 + g + 8 * r;
     qpos[r] = row < n ? lens[row] - 1 : 0;
   }
-  const int nb = (S + BKV - 1) / BKV;
+  issue(0);  // also completes the Q copies (same commit group)
   for (int kb = 0; kb < nb; ++kb) {
-    const int kbase = kb * BKV, kcount = min(BKV, S - kbase);
-    __syncthreads();
-    for (int c = tid; c < BKV * (DH / 8); c += 128) {
-      const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
-      const bool ok = row < kcount;
-      const int key = kbase + row;
-      const T* src = pool;
-      if (ok) src = pool + (size_t)prow[key / PAGE] * page_elems + ((size_t)hk * PAGE + key % PAGE) * DH + col;
-      cp_async16(sK + row * LD + col, src, ok);
-      cp_async16(sV + row * LD + col, ok ? src + v_off : pool, ok);
+    if (kb + 1 < nb) {
+      issue(kb + 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
     }
-    cp_async_wait_all();
     __syncthreads();
+    const T* sK = sKV + (size_t)(kb & 1) * 2 * BKV * LD;
+    const T* sV = sK + BKV * LD;
+    const int kbase = kb * BKV, kcount = min(BKV, S - kbase);
     float sc[BKV / 8][4];
 #pragma unroll
     for (int i = 0; i < BKV / 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
@@ -688,24 +726,8 @@ __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, co
       o[i][0] *= corr[0], o[i][1] *= corr[0];
       o[i][2] *= corr[1], o[i][3] *= corr[1];
     }
-#pragma unroll
-    for (int kk = 0; kk < BKV / 16; ++kk) {
-      uint32_t ah[4], al[4];
-      split16<T>(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
-      split16<T>(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
-      split16<T>(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
-      split16<T>(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
-#pragma unroll
-      for (int dp = 0; dp < DH / 16; ++dp) {
-        uint32_t b0, b1, b2, b3;
-        ldm_x4_t(smem_addr(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LD + dp * 16 + (lane >> 4) * 8), b0,
-                 b1, b2, b3);
-        mma16816<T>(o[2 * dp], ah[0], ah[1], ah[2], ah[3], b0, b1);
-        mma16816<T>(o[2 * dp + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
-        mma16816<T>(o[2 * dp], al[0], al[1], al[2], al[3], b0, b1);
-        mma16816<T>(o[2 * dp + 1], al[0], al[1], al[2], al[3], b2, b3);
-      }
-    }
+    pv_accumulate<T, DH / 16>(sc, sV, LD, lane, o);
+    __syncthreads();  // this stage is refilled by the next iteration's issue
   }
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
@@ -714,7 +736,7 @@ __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, co
   }
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
-    const int row = s0 + warp * 16 + g + 8 * r;
+    const int row = s0 + g + 8 * r;
     if (row >= n) continue;
     float* pp = part + ((size_t)row * Hq + hq) * max_splits * (DH + 2);   // partial slot 0
 #pragma unroll
@@ -786,14 +808,15 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
   const int t_min = shared_pos;
   if (sbase) {
     if (!part) return set_err(SR_ERR_INVALID_ARG, "decode attention: partial buffer missing for the prefix pass");
-    const size_t psmem = (size_t)(BQ + 2 * BKV) * (DH + 8) * sizeof(T);
+    constexpr int HPC = G < 4 ? G : 4, CPC = 4 / HPC;
+    const size_t psmem = (size_t)(BQ + 4 * BKV) * (DH + 8) * sizeof(T);
     static bool pattr = false;
     if (!pattr) {
-      SR_CUDA(cudaFuncSetAttribute(k_prefix_attn<T, DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem));
+      SR_CUDA(cudaFuncSetAttribute(k_prefix_attn<T, DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem));
       pattr = true;
     }
-    k_prefix_attn<T, DH><<<dim3((b + BQ - 1) / BQ, Hkv * G), 128, psmem, st>>>(
-        (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, b, shared_pos, Hkv * G, Hkv,
+    k_prefix_attn<T, DH, G><<<dim3((b + 16 * CPC - 1) / (16 * CPC), Hkv * (G / HPC)), 128, psmem, st>>>(
+        (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, b, shared_pos, Hkv,
         1.4426950408889634f / sqrtf((float)DH), window, max_splits, part);
     SR_LAUNCH();
   }
