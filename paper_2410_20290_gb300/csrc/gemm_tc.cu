@@ -22,6 +22,8 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+#include <cmath>
 #include <cstdlib>
 #include <mutex>
 
@@ -30,18 +32,24 @@
 namespace sr {
 namespace {
 
-constexpr int BM = 128, BK = 64;
-constexpr int A_BYTES = BM * BK * 2;  // 16 KB
-constexpr int NUM_THREADS = 192;
+constexpr int BM = 128, BK = 64;  // BM: rows of one MMA (one TMEM lane block)
 constexpr int BAR_BYTES = 256;
 constexpr unsigned long long WAIT_NS = 2000000000ull;
 
-template <int BN>
+// TM = rows per CTA tile: 128 (one MMA per K step) or 256 (two MMAs sharing the W tile, which halves the
+// staged bytes per flop; its 256 x 256 fp32 accumulator fills TMEM, so it is single-buffered and drained
+// by eight epilogue warps instead of four).
+template <int TM, int BN>
 struct Cfg {
+  static constexpr int MH = TM / BM;                          // 128-row halves per tile
+  static constexpr int A_BYTES = TM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (192 * 1024) / STAGE_BYTES;  // 4 / 6 / 8 stages for BN 256 / 128 / 64
-  static constexpr int TMEM_COLS = 2 * BN;                   // two accumulators
+  static constexpr int STAGES = (192 * 1024) / STAGE_BYTES;  // 4 / 6 / 8 for BN 256 / 128 / 64; 3 for 256 x 256
+  static constexpr int NACC = (MH * BN * 2 <= 512) ? 2 : 1;   // accumulator buffers in TMEM
+  static constexpr int TMEM_COLS = NACC * MH * BN;
+  static constexpr int EPI_WARPS = 4 * MH;
+  static constexpr int THREADS = 64 + 32 * EPI_WARPS;
   static constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
 };
 
@@ -118,6 +126,30 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
+// commit that arrives on the barrier at this smem offset in every CTA of `mask` in the cluster
+__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "h"(mask)
+               : "memory");
+}
+// 2D TMA load written to the same smem offset in every CTA of `mask`, signalling each CTA's barrier
+__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
+                                               uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, "
+      "{%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -169,12 +201,20 @@ struct EpiArgs {
   int bf;   // operands and 16-bit outputs are bf16 (1) or fp16 (0)
 };
 
-template <int BN>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+// CL = 2: the kernel runs in clusters of two CTAs that take the two M tiles of a pair with the same W
+// tile; each CTA loads half of the W tile and multicasts it to both, so the L2 -> SM traffic per stage
+// drops from 48 KB to 32 KB (BN = 256).  Stage release is signalled to both CTAs (empty barriers count
+// two commits).  When the M-tile count is odd, the last pair's second tile is all zero-filled rows that
+// the epilogue skips.
+template <int TM, int BN, int CL>
+__global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
               int N, int K, int* err) {
-  constexpr int B_BYTES = Cfg<BN>::B_BYTES, STAGE_BYTES = Cfg<BN>::STAGE_BYTES, STAGES = Cfg<BN>::STAGES;
-  constexpr int TMEM_COLS = Cfg<BN>::TMEM_COLS;
+  using C = Cfg<TM, BN>;
+  constexpr int A_BYTES = C::A_BYTES, B_BYTES = C::B_BYTES, STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES;
+  constexpr int TMEM_COLS = C::TMEM_COLS, MH = C::MH, NACC = C::NACC, EPI_WARPS = C::EPI_WARPS;
+  constexpr int ACC_COLS = MH * BN;  // TMEM columns of one accumulator buffer
+  static_assert(CL == 1 || CL == 2, "cluster size");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -189,17 +229,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t idesc = idesc_for(ep.bf != 0, BN);
-  const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN, num_tiles = num_m * num_n;
+  const int num_m = (M + TM - 1) / TM, num_n = (N + BN - 1) / BN;
   const int num_k = (K + BK - 1) / BK;
+  // tiles of this CTA: index t over (M-tile group of CL, N tile), M fastest; m tile = CL * group + rank
+  const int rank = CL == 2 ? (int)cluster_rank() : 0;
+  const int num_mg = (num_m + CL - 1) / CL, num_tiles = num_mg * num_n;
+  const int t0 = blockIdx.x / CL, tstep = gridDim.x / CL;
+  constexpr uint16_t MASK = CL == 2 ? 0x3 : 0x1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], CL);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], EPI_WARPS);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -214,6 +259,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if (CL == 2) cluster_sync();  // the peer's barriers are initialised before anyone signals them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -226,16 +272,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t armed_par[STAGES];
       for (int s = 0; s < STAGES; ++s) armed[s] = 0, armed_par[s] = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        const int mb = tile % num_m, nb = tile / num_m;
+      for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
+        const int mb = (tile % num_mg) * CL + rank, nb = tile / num_mg;
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
             ok = false;
             break;
           }
           mbar_expect_tx(&full[stage], STAGE_BYTES);
-          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * BM);
-          tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * BN);
+          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * TM);
+          if (CL == 2)
+            tma_load_2d_mc(sB + stage * B_BYTES + rank * (B_BYTES / 2), &tmB, &full[stage], kb * BK,
+                           nb * BN + rank * (BN / 2), MASK);
+          else
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * BN);
           armed[stage] = 1;
           armed_par[stage] = phase;
           if (++stage == STAGES) stage = 0, phase ^= 1u;
@@ -257,30 +307,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * ACC_COLS);
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint64_t a0 = sdesc(smem_u32(sA + stage * A_BYTES));
           const uint64_t b0 = sdesc(smem_u32(sB + stage * B_BYTES));
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes per K=16 step inside the swizzle atom
-            umma(d_tmem, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc, (kb | kk) != 0);
-          umma_commit(&empty[stage]);
+          for (int h = 0; h < MH; ++h) {  // 128-row halves of the tile share the W tile
+            const uint64_t a0 = sdesc(smem_u32(sA + stage * A_BYTES + h * (BM * BK * 2)));
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes per K=16 step inside the swizzle atom
+              umma(d_tmem + (uint32_t)(h * BN), a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc,
+                   (kb | kk) != 0);
+          }
+          if (CL == 2) umma_commit_mc(&empty[stage], MASK);
+          else umma_commit(&empty[stage]);
           if (++stage == STAGES) stage = 0, phase ^= 1u;
         }
         if (!ok) break;
         umma_commit(&tfull[acc]);
-        if (++acc == 2) acc = 0, acc_phase ^= 1u;
+        if (++acc == NACC) acc = 0, acc_phase ^= 1u;
       }
       if (!ok) {
         atomicExch(err, 2);
@@ -291,12 +346,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_wait(mma_done, 0, nullptr);
     }
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int quad = warp & 3;
+    // ---------------- epilogue (warps 2 .. 2 + EPI_WARPS) ----------------
+    // warp w reads TMEM lane quadrant w % 4 (the hardware's lane-access rule) of half (w - 2) / 4
+    const int quad = warp & 3, half = (warp - 2) / 4;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-      const int mb = tile % num_m, nb = tile / num_m;
+    for (int tile = t0; tile < num_tiles; tile += tstep) {
+      const int mb = (tile % num_mg) * CL + rank, nb = tile / num_mg;
       // one lane waits and broadcasts, so the warp-collective tcgen05.ld below stays converged
       int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag) : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -308,8 +364,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         break;
       }
       tc_fence_after();
-      const int row = mb * BM + quad * 32 + lane;
-      const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
+      const int row = mb * TM + half * BM + quad * 32 + lane;
+      const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * ACC_COLS + half * BN);
       const int col0 = nb * BN;
       if (ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU) {
 #pragma unroll 1
@@ -357,11 +413,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
-      if (++acc == 2) acc = 0, acc_phase ^= 1u;
+      if (++acc == NACC) acc = 0, acc_phase ^= 1u;
     }
   }
   tc_fence_before();
   __syncthreads();
+  if (CL == 2) cluster_sync();  // no peer still writes into this CTA's shared memory or barriers
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
@@ -372,6 +429,8 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 int g_num_sms = 0;
 int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
+int g_cl_override = 0;  // SR_GEMM_CL: force the cluster size (1 or 2)
+int g_tm_override = 0;  // SR_GEMM_TM: force the tile height (128 or 256)
 int* g_err = nullptr;
 
 // Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost.  The per-tile
@@ -391,18 +450,59 @@ int pick_bn(int M, int N, int K) {
   return best;
 }
 
-template <int BN>
+// Tall 256 x 256 tiles pay when they keep the SMs about as busy as the 128-row tiles: compare waves x
+// per-tile cost, a 256 x 256 tile costing about 1.5 128 x 256 tiles (twice the MMA work at the higher
+// tensor-pipe occupancy its halved staging allows).
+bool pick_tall(int M, int N, int K) {
+  (void)K;
+  if (M < 2 * BM) return false;
+  const int bn = pick_bn(M, N, K);
+  const double t_small = std::ceil((double)((M + BM - 1) / BM) * ((N + bn - 1) / bn) / g_num_sms) *
+                         (bn * (K / 4096.0) + 430.0);
+  const double t_tall = std::ceil((double)((M + 255) / 256) * ((N + 255) / 256) / g_num_sms) * 1.5 *
+                        (256 * (K / 4096.0) + 430.0);
+  return t_tall < t_small;
+}
+
+template <int TM, int BN, int CL>
 sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
                     cudaStream_t st) {
-  static bool attr = false;
-  if (!attr) {
-    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::SMEM_BYTES));
-    attr = true;
+  using C = Cfg<TM, BN>;
+  static int max_groups = 0;
+  if (!max_groups) {
+    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 C::SMEM_BYTES));
+    max_groups = g_num_sms / CL;
+    if (CL > 1) {
+      SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN, CL>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0));
+      cudaLaunchConfig_t qc = {};
+      cudaLaunchAttribute qa[1];
+      qa[0].id = cudaLaunchAttributeClusterDimension;
+      qa[0].val.clusterDim.x = CL, qa[0].val.clusterDim.y = 1, qa[0].val.clusterDim.z = 1;
+      qc.gridDim = dim3(g_num_sms / CL * CL);
+      qc.blockDim = dim3(C::THREADS);
+      qc.dynamicSmemBytes = C::SMEM_BYTES;
+      qc.attrs = qa;
+      qc.numAttrs = 1;
+      int clusters = 0;
+      if (cudaOccupancyMaxActiveClusters(&clusters, k_gemm_tc<TM, BN, CL>, &qc) == cudaSuccess && clusters > 0)
+        max_groups = std::min(max_groups, clusters);
+      cudaGetLastError();
+    }
   }
-  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
-  k_gemm_tc<BN><<<grid, NUM_THREADS, Cfg<BN>::SMEM_BYTES, st>>>(ta, tb, ep, M, N, K, g_err);
-  SR_LAUNCH();
+  const int groups_total = ((M + TM * CL - 1) / (TM * CL)) * ((N + BN - 1) / BN);
+  const int groups = std::min(groups_total, max_groups);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL, attr[0].val.clusterDim.y = 1, attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(groups * CL);
+  cfg.blockDim = dim3(C::THREADS);
+  cfg.dynamicSmemBytes = C::SMEM_BYTES;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  SR_CUDA(cudaLaunchKernelEx(&cfg, k_gemm_tc<TM, BN, CL>, ta, tb, ep, M, N, K, g_err));
   return SR_OK;
 }
 
@@ -445,16 +545,30 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     SR_CUDA(cudaMalloc(&g_err, sizeof(int)));
     SR_CUDA(cudaMemset(g_err, 0, sizeof(int)));
     if (const char* e = getenv("SR_GEMM_BN")) g_bn_override = atoi(e);
+    if (const char* e = getenv("SR_GEMM_CL")) g_cl_override = atoi(e);
+    if (const char* e = getenv("SR_GEMM_TM")) g_tm_override = atoi(e);
   }
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
-  const int bn = pick_bn(M, N, K);
+  int tm = 128, bn = pick_bn(M, N, K);
+  // (gated epilogues are the longest, and the single-buffered tall tile cannot hide them: 128-row tiles there)
+  if (g_tm_override == 256 || (g_tm_override == 0 && g_bn_override == 0 && !gated && pick_tall(M, N, K)))
+    tm = 256, bn = 256;
+  // cluster multicast of the W tile across two M tiles (measured neutral on GB300; kept selectable)
+  const int cl = g_cl_override == 2 ? 2 : 1;
   CUtensorMap ta, tb;
-  SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
-  SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn));
+  SR_TRY(encode_kmajor(&ta, A, bf, M, K, tm));
+  SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn / cl));
   EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
-  if (bn == 64) return launch_bn<64>(ta, tb, ep, M, N, K, st);
-  if (bn == 128) return launch_bn<128>(ta, tb, ep, M, N, K, st);
-  return launch_bn<256>(ta, tb, ep, M, N, K, st);
+  if (tm == 256) return cl == 2 ? launch_bn<256, 256, 2>(ta, tb, ep, M, N, K, st)
+                                : launch_bn<256, 256, 1>(ta, tb, ep, M, N, K, st);
+  if (cl == 2) {
+    if (bn == 64) return launch_bn<128, 64, 2>(ta, tb, ep, M, N, K, st);
+    if (bn == 128) return launch_bn<128, 128, 2>(ta, tb, ep, M, N, K, st);
+    return launch_bn<128, 256, 2>(ta, tb, ep, M, N, K, st);
+  }
+  if (bn == 64) return launch_bn<128, 64, 1>(ta, tb, ep, M, N, K, st);
+  if (bn == 128) return launch_bn<128, 128, 1>(ta, tb, ep, M, N, K, st);
+  return launch_bn<128, 256, 1>(ta, tb, ep, M, N, K, st);
 }
 
 // Device error word of the tensor-core GEMM (nonzero after a bounded wait expired).

@@ -1,0 +1,26 @@
+"""The tcgen05 GEMM's alternative tile shapes, checked with the same GEMM cases as the default launch.
+
+The launcher reads its tile overrides (SR_GEMM_TM: 256-row tiles with two MMAs per W tile;
+SR_GEMM_CL: two-CTA clusters sharing the W tile by multicast) once per process, so each variant
+runs the GEMM cases of test_gpu_kernels.py in a child process of its own.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.mark.parametrize("env", [{"SR_GEMM_TM": "256"}, {"SR_GEMM_CL": "2"}, {"SR_GEMM_TM": "256", "SR_GEMM_CL": "2"},
+                                 {"SR_GEMM_BN": "64"}, {"SR_GEMM_BN": "128"}])
+def test_gemm_tile_variant(env):
+    child = dict(os.environ, **env)
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-m", "gpu", "-k", "gemm_tc", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_gpu_kernels.py")], cwd=ROOT, env=child,
+                       capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout[-4000:] + r.stderr[-2000:]
+    assert " passed" in r.stdout and "skipped" not in r.stdout.split("\n")[-2]
