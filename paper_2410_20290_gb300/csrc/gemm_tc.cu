@@ -17,6 +17,10 @@
 //                 direct global stores
 // Two BN-column accumulators let the epilogue of tile i overlap the mainloop of tile i+1.
 // Tiles are walked M-fastest so that the CTAs running at the same time share W tiles in L2.
+// Two variants raise the MMA work per staged byte (the limit of the 128-row tiles on GB300):
+// 256 x 256 tiles on one SM (two M = 128 MMAs per W tile, single-buffered accumulator), and
+// 256 x 256 tiles on a CTA pair (cta_group::2, M = 256 MMAs, each SM staging half of A and W,
+// double-buffered accumulators).  The launcher picks among the three per shape.
 // Every mbarrier wait is bounded (about 2 s of %globaltimer); on expiry the CTA records an error,
 // drains its own TMA copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
@@ -201,6 +205,118 @@ struct EpiArgs {
   int bf;   // operands and 16-bit outputs are bf16 (1) or fp16 (0)
 };
 
+// ---- CTA-pair (cta_group::2) forms ----
+// Wait whose phase is completed by arrivals from the peer CTA: acquire at cluster scope.
+__device__ __forceinline__ bool mbar_test_cl(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __noinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  const uint32_t addr = smem_u32(bar);
+  if (mbar_test_cl(addr, parity)) return true;
+  const unsigned long long t0 = gtimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_test_cl(addr, parity)) return true;
+    if (abort_flag && *abort_flag) return false;
+    if (gtimer() - t0 > WAIT_NS) return false;
+  }
+}
+// Address of the barrier at this smem offset in CTA `cta` of the cluster.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t cta) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(p)), "r"(cta));
+  return remote;
+}
+// Arrive on the barrier at this smem offset in CTA `cta` of the cluster (release at cluster scope).
+__device__ __forceinline__ void mbar_arrive_cta(uint64_t* bar, uint32_t cta) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr(bar, cta))
+               : "memory");
+}
+// 2D TMA load into this CTA's shared memory whose completion (complete_tx) is counted on a barrier of
+// either CTA of the pair (`bar_cluster`, a shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar_cluster, int x,
+                                                 int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+// One M = 256 MMA over the pair: A rows 0-127 and W rows 0 .. N/2-1 from the issuing CTA's shared
+// memory, A rows 128-255 and W rows N/2 .. N-1 from the same offsets in the peer's; each CTA's TMEM
+// receives its 128 rows x N columns.
+__device__ __forceinline__ void umma_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
+}
+__device__ __forceinline__ void umma_pair_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "h"(mask)
+               : "memory");
+}
+
+// Epilogue of one accumulator row segment: this thread's row of BNC fp32 columns at TMEM address
+// `tbase`, converted / activated / added and stored at (row, col0 ..).  Rows >= M and columns >= N are
+// skipped (they hold the zero-filled tails of the TMA tiles).
+template <int BNC>
+__device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int row, int col0, int M, int N) {
+  if (ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU) {
+#pragma unroll 1
+    for (int c = 0; c < BNC; c += 64) {
+      float g[32], u[32];
+      tmem_ld16(tbase + c, g);
+      tmem_ld16(tbase + c + 16, g + 16);
+      tmem_ld16(tbase + c + 32, u);
+      tmem_ld16(tbase + c + 48, u + 16);
+      if (row < M && col0 + c < N) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) g[j] = (ep.kind == EPI_SWIGLU ? silu_f(g[j]) : gelu_f(g[j])) * u[j];
+        uint16_t* dst = reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + (col0 + c) / 2;
+        store16x32(dst, g, ep.bf != 0);
+      }
+    }
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < BNC; c += 32) {
+      float v[32];
+      tmem_ld16(tbase + c, v);
+      tmem_ld16(tbase + c + 16, v + 16);
+      if (row < M && col0 + c < N) {
+        if (ep.kind == EPI_F32 || ep.kind == EPI_ADD_F32) {
+          float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)row * ep.ldo + col0 + c);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            if (ep.kind == EPI_ADD_F32) {
+              const float4 r = dst[q];
+              o.x += r.x, o.y += r.y, o.z += r.z, o.w += r.w;
+            }
+            dst[q] = o;
+          }
+        } else {
+          if (ep.kind == EPI_GELU) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
+          }
+          store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col0 + c, v, ep.bf != 0);
+        }
+      }
+    }
+  }
+}
+
 // CL = 2: the kernel runs in clusters of two CTAs that take the two M tiles of a pair with the same W
 // tile; each CTA loads half of the W tile and multicasts it to both, so the L2 -> SM traffic per stage
 // drops from 48 KB to 32 KB (BN = 256).  Stage release is signalled to both CTAs (empty barriers count
@@ -366,50 +482,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       tc_fence_after();
       const int row = mb * TM + half * BM + quad * 32 + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * ACC_COLS + half * BN);
-      const int col0 = nb * BN;
-      if (ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU) {
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 64) {
-          float g[32], u[32];
-          tmem_ld16(tbase + c, g);
-          tmem_ld16(tbase + c + 16, g + 16);
-          tmem_ld16(tbase + c + 32, u);
-          tmem_ld16(tbase + c + 48, u + 16);
-          if (row < M && col0 + c < N) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) g[j] = (ep.kind == EPI_SWIGLU ? silu_f(g[j]) : gelu_f(g[j])) * u[j];
-            uint16_t* dst = reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + (col0 + c) / 2;
-            store16x32(dst, g, ep.bf != 0);
-          }
-        }
-      } else {
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          float v[32];
-          tmem_ld16(tbase + c, v);
-          tmem_ld16(tbase + c + 16, v + 16);
-          if (row < M && col0 + c < N) {
-            if (ep.kind == EPI_F32 || ep.kind == EPI_ADD_F32) {
-              float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)row * ep.ldo + col0 + c);
-#pragma unroll
-              for (int q = 0; q < 8; ++q) {
-                float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                if (ep.kind == EPI_ADD_F32) {
-                  const float4 r = dst[q];
-                  o.x += r.x, o.y += r.y, o.z += r.z, o.w += r.w;
-                }
-                dst[q] = o;
-              }
-            } else {
-              if (ep.kind == EPI_GELU) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
-              }
-              store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col0 + c, v, ep.bf != 0);
-            }
-          }
-        }
-      }
+      epi_store<BN>(ep, tbase, row, nb * BN, M, N);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -425,12 +498,211 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------------------------------------
+// CTA-pair GEMM (cta_group::2): clusters of two CTAs on two SMs compute one 256 x BNP tile with
+// M = 256 MMAs issued by the even CTA.  Each CTA stages only its own 128 rows of A and BNP/2 rows of
+// W per K block (32 KB for BNP = 256: 128 flop per staged byte, against 85 for a 128 x 256 tile on
+// one SM), so six stages fit, and each CTA's TMEM holds its 128 x BNP share of two accumulators,
+// keeping the epilogue overlapped with the next tile's mainloop.
+//   warp 0 (both CTAs) : TMA of the CTA's own A and W halves into its own shared memory; both CTAs'
+//                        copies complete on the even CTA's full barrier, which expects both
+//   warp 1, even CTA   : issues the MMAs, commits stage release and accumulator-ready to both CTAs
+//   warps 2-5 (both)   : epilogue of the CTA's 128 rows; arrive on the even CTA's tempty barrier
+// Every wait is bounded.  On abort the even CTA drains the stages it armed (their phases count both
+// CTAs' copies); the odd CTA, whose copies complete on the other CTA's barriers, waits 1 ms for its
+// own copies in flight before it leaves.
+template <int BNP>
+struct PairCfg {
+  static constexpr int A_BYTES = BM * BK * 2;             // 16 KB
+  static constexpr int B_BYTES = (BNP / 2) * BK * 2;      // 16 KB for BNP = 256
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = (192 * 1024) / STAGE_BYTES;
+  static constexpr int TMEM_COLS = 2 * BNP;
+  static constexpr int THREADS = 192;
+  static constexpr int GUARD = 32 * 1024;  // keeps any operand read of the last stage inside the allocation
+  static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + GUARD + BAR_BYTES;
+};
+
+__host__ __device__ constexpr uint32_t idesc_pair(bool bf, int N) {
+  return (1u << 4) | ((bf ? 1u : 0u) << 7) | ((bf ? 1u : 0u) << 10) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(256 >> 4) << 24);
+}
+
+template <int BNP>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
+    k_gemm_pair(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
+                int N, int K, int* err) {
+  using C = PairCfg<BNP>;
+  constexpr int A_BYTES = C::A_BYTES, B_BYTES = C::B_BYTES, STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES;
+  constexpr int TMEM_COLS = C::TMEM_COLS;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + C::GUARD);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const uint32_t idesc = idesc_pair(ep.bf != 0, BNP);
+  const int num_m = (M + 255) / 256, num_n = (N + BNP - 1) / BNP;
+  const int num_k = (K + BK - 1) / BK;
+  const int num_tiles = num_m * num_n;
+  const int t0 = blockIdx.x / 2, tstep = gridDim.x / 2;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 8);  // four epilogue warps in each CTA
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs' barriers are initialised (and TMEM allocated) before any cross-CTA signal
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (own halves) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int armed[STAGES];
+      uint32_t armed_par[STAGES];
+      for (int s = 0; s < STAGES; ++s) armed[s] = 0, armed_par[s] = 0;
+      bool ok = true;
+      for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
+        const int mb = tile % num_m, nb = tile / num_m;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          // the even CTA's barrier counts both CTAs' bytes; the odd CTA's copies may land first (the
+          // transaction count goes negative until the expect_tx, and the phase cannot complete before it)
+          if (rank == 0) mbar_expect_tx(&full[stage], 2 * STAGE_BYTES);
+          const uint32_t bar = cluster_addr(&full[stage], 0);
+          tma_load_2d_pair(sA + stage * A_BYTES, &tmA, bar, kb * BK, mb * 256 + (int)rank * BM);
+          tma_load_2d_pair(sB + stage * B_BYTES, &tmB, bar, kb * BK, nb * BNP + (int)rank * (BNP / 2));
+          armed[stage] = 1;
+          armed_par[stage] = phase;
+          if (++stage == STAGES) stage = 0, phase ^= 1u;
+        }
+      }
+      if (!ok) {
+        atomicExch(err, 1);
+        *abort_flag = 1;
+        if (rank == 0) {
+          for (int s = 0; s < STAGES; ++s)
+            if (armed[s]) mbar_wait(&full[s], armed_par[s], nullptr);
+        } else {
+          const unsigned long long t = gtimer();
+          while (gtimer() - t < 1000000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---------------- MMA issuer (even CTA) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
+        if (!mbar_wait_cl(&tempty[acc], acc_phase ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BNP);
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t a0 = sdesc(smem_u32(sA + stage * A_BYTES));
+          const uint64_t b0 = sdesc(smem_u32(sB + stage * B_BYTES));
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            umma_pair(d_tmem, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc, (kb | kk) != 0);
+          umma_pair_commit_mc(&empty[stage], 0x3);
+          if (++stage == STAGES) stage = 0, phase ^= 1u;
+        }
+        if (!ok) break;
+        umma_pair_commit_mc(&tfull[acc], 0x3);
+        if (++acc == 2) acc = 0, acc_phase ^= 1u;
+      }
+      if (!ok) {
+        atomicExch(err, 2);
+        *abort_flag = 1;
+      }
+      umma_pair_commit_mc(mma_done, 0x1);
+      mbar_wait(mma_done, 0, nullptr);
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 of both CTAs) ----------------
+    const int quad = warp & 3;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = t0; tile < num_tiles; tile += tstep) {
+      const int mb = tile % num_m, nb = tile / num_m;
+      int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag) : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          atomicExch(err, 3);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const int row = mb * 256 + (int)rank * BM + quad * 32 + lane;
+      const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BNP);
+      epi_store<BNP>(ep, tbase, row, nb * BNP, M, N);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cta(&tempty[acc], 0);
+      if (++acc == 2) acc = 0, acc_phase ^= 1u;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the even CTA's MMAs are complete and no CTA signals the other any more
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 int g_num_sms = 0;
 int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
 int g_cl_override = 0;  // SR_GEMM_CL: force the cluster size (1 or 2)
 int g_tm_override = 0;  // SR_GEMM_TM: force the tile height (128 or 256)
+int g_pair_override = -1;  // SR_GEMM_PAIR: 1 forces the CTA-pair kernel, 0 forbids it
 int* g_err = nullptr;
 
 // Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost.  The per-tile
@@ -506,6 +778,38 @@ sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs&
   return SR_OK;
 }
 
+// Where the CTA-pair kernel measured faster on GB300 than the one-SM tiles: gated epilogues (its
+// double-buffered accumulator hides them), LM-head widths, and down-projection shapes (N <= 4096,
+// K >= 8192) below 8192 rows; at least two pair rows (M >= 512) so the 256-row tiles are not mostly padding.
+bool pick_pair(int M, int N, int K, bool gated) {
+  if (M < 512) return false;
+  return gated || N >= 65536 || (N <= 4096 && K >= 8192 && M < 8192);
+}
+
+template <int BNP>
+sr_status launch_pair(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
+                      cudaStream_t st) {
+  using C = PairCfg<BNP>;
+  static int max_pairs = 0;
+  if (!max_pairs) {
+    SR_CUDA(cudaFuncSetAttribute(k_gemm_pair<BNP>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
+    max_pairs = g_num_sms / 2;
+    cudaLaunchConfig_t qc = {};
+    qc.gridDim = dim3(max_pairs * 2);
+    qc.blockDim = dim3(C::THREADS);
+    qc.dynamicSmemBytes = C::SMEM_BYTES;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, k_gemm_pair<BNP>, &qc) == cudaSuccess && clusters > 0)
+      max_pairs = std::min(max_pairs, clusters);
+    cudaGetLastError();
+  }
+  const int tiles = ((M + 255) / 256) * ((N + BNP - 1) / BNP);
+  const int pairs = std::min(tiles, max_pairs);
+  k_gemm_pair<BNP><<<pairs * 2, C::THREADS, C::SMEM_BYTES, st>>>(ta, tb, ep, M, N, K, g_err);
+  SR_CUDA(cudaGetLastError());
+  return SR_OK;
+}
+
 sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, int K, int box_rows) {
   std::call_once(g_encode_once, [] {
     void* fn = nullptr;
@@ -547,18 +851,25 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     if (const char* e = getenv("SR_GEMM_BN")) g_bn_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_CL")) g_cl_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_TM")) g_tm_override = atoi(e);
+    if (const char* e = getenv("SR_GEMM_PAIR")) g_pair_override = atoi(e);
   }
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
+  CUtensorMap ta, tb;
+  EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
+  if (g_pair_override == 1 || (g_pair_override == -1 && g_bn_override == 0 && g_tm_override == 0 &&
+                               g_cl_override == 0 && pick_pair(M, N, K, gated))) {
+    SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
+    SR_TRY(encode_kmajor(&tb, W, bf, N, K, 128));
+    return launch_pair<256>(ta, tb, ep, M, N, K, st);
+  }
   int tm = 128, bn = pick_bn(M, N, K);
   // (gated epilogues are the longest, and the single-buffered tall tile cannot hide them: 128-row tiles there)
   if (g_tm_override == 256 || (g_tm_override == 0 && g_bn_override == 0 && !gated && pick_tall(M, N, K)))
     tm = 256, bn = 256;
   // cluster multicast of the W tile across two M tiles (measured neutral on GB300; kept selectable)
   const int cl = g_cl_override == 2 ? 2 : 1;
-  CUtensorMap ta, tb;
   SR_TRY(encode_kmajor(&ta, A, bf, M, K, tm));
   SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn / cl));
-  EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
   if (tm == 256) return cl == 2 ? launch_bn<256, 256, 2>(ta, tb, ep, M, N, K, st)
                                 : launch_bn<256, 256, 1>(ta, tb, ep, M, N, K, st);
   if (cl == 2) {

@@ -1,7 +1,8 @@
 """The tcgen05 GEMM's alternative tile shapes, checked with the same GEMM cases as the default launch.
 
-The launcher reads its tile overrides (SR_GEMM_TM: 256-row tiles with two MMAs per W tile;
-SR_GEMM_CL: two-CTA clusters sharing the W tile by multicast) once per process, so each variant
+The launcher reads its tile overrides (SR_GEMM_PAIR: 256 x 256 tiles computed by a CTA pair with
+cta_group::2 MMAs; SR_GEMM_TM: 256-row tiles with two MMAs per W tile on one SM; SR_GEMM_CL: two-CTA
+clusters sharing the W tile by multicast) once per process, so each variant
 runs the GEMM cases of test_gpu_kernels.py in a child process of its own.
 """
 import os
@@ -15,8 +16,8 @@ pytestmark = pytest.mark.gpu
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-@pytest.mark.parametrize("env", [{"SR_GEMM_TM": "256"}, {"SR_GEMM_CL": "2"}, {"SR_GEMM_TM": "256", "SR_GEMM_CL": "2"},
-                                 {"SR_GEMM_BN": "64"}, {"SR_GEMM_BN": "128"}])
+@pytest.mark.parametrize("env", [{"SR_GEMM_PAIR": "1"}, {"SR_GEMM_TM": "256"}, {"SR_GEMM_CL": "2"},
+                                 {"SR_GEMM_TM": "256", "SR_GEMM_CL": "2"}, {"SR_GEMM_BN": "64"}, {"SR_GEMM_BN": "128"}])
 def test_gemm_tile_variant(env):
     child = dict(os.environ, **env)
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-m", "gpu", "-k", "gemm_tc", "-p", "no:cacheprovider",
