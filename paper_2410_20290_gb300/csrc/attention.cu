@@ -143,8 +143,9 @@ __global__ void k_decode_combine(const float* __restrict__ part, const int* __re
   const int hq = blockIdx.x, s = blockIdx.y, d = threadIdx.x;
   const int L = lens[s];
   const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
-  const int total = sbase + (L - t_lo + SPLIT - 1) / SPLIT;
-  if (total <= 1) return;  // written directly by the attention kernel
+  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  if (nsplit <= 1 && (sbase == 0 || nsplit == 1)) return;  // written directly by the attention kernel
+  const int total = sbase + nsplit;
   const float* pp = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
   float M = -INFINITY;
   for (int j = 0; j < total; ++j) M = fmaxf(M, pp[j * (DH + 2) + DH]);
@@ -398,7 +399,14 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       O += so[((size_t)w * DH + d) * 8 + j] * wt;
     }
     const int hq = h * G + j;
-    if (nsplit == 1 && sbase == 0) {
+    if (nsplit == 1) {
+      if (sbase) {  // fold in the shared-prefix pass (partial slot 0, written by the preceding launch)
+        const float* p0 = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
+        const float m0 = p0[DH], Mn = fmaxf(M, m0);
+        const float w0 = (m0 == -INFINITY) ? 0.f : exp2f(m0 - Mn), w1 = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
+        O = O * w1 + p0[d] * w0;
+        Lsum = Lsum * w1 + p0[DH + 1] * w0;
+      }
       out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
     } else {
       float* pp = part + (((size_t)s * Hq + hq) * max_splits + sbase + split) * (DH + 2);
@@ -598,7 +606,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
 // several candidates for up to 4 query heads of one kv head (64 query rows, one warp per 16 rows) and runs
 // flash attention over the prefix keys with mma.sync; each 64-position K/V block is loaded once per CTA
 // through a 2-stage cp.async pipeline.  The result is written unnormalised as partial slot 0 (O, m, l in
-// the decode kernels' log2-scaled convention) for k_decode_combine to merge with the suffix partials.
+// the decode kernels' log2-scaled convention); the suffix kernel folds it into its result when a row's
+// suffix is one split, k_decode_combine merges it with the split partials otherwise.
 // No causal mask is needed (every prefix position precedes the query); a window masks per row.
 template <typename T, int DH, int G>
 __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, const T* __restrict__ pool,
@@ -833,7 +842,7 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
   k_decode_attn_tc<T, DH, G><<<grid, 128, smem, st>>>((const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
                                                        scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
   SR_LAUNCH();
-  if (max_splits > 1) {
+  if (max_splits - sbase > 1) {  // some row has several position splits (a lone split merges the prefix itself)
     k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, t_min, sbase,
                                                              (T*)out);
     SR_LAUNCH();

@@ -5,6 +5,8 @@
 // These compute the per-position parts of the generator and reward model of Section 3; the KV
 // append is the paged cache of the Section 5 engine ("pre-allocates the corresponding KV cache").
 #include <algorithm>
+#include <cstdint>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -48,6 +50,70 @@ __global__ void k_norm(const float* __restrict__ x, const T* __restrict__ w, con
     float v = (xr[c] - mean) * rstd * to_f(w[c]);
     if (layer_norm) v += to_f(b[c]);
     orow[c] = f_to<T>(v);
+  }
+}
+
+// Vectorised form for d % 4 == 0 and d <= 16 * blockDim.x: the row stays in registers (up to four
+// float4 per thread, consecutive float4 across a warp), one pass over x.
+template <typename T>
+__device__ __forceinline__ void store4(T* p, float a, float b, float c, float d) {
+  if constexpr (std::is_same<T, float>::value) {
+    *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+  } else {
+    T h[4] = {f_to<T>(a), f_to<T>(b), f_to<T>(c), f_to<T>(d)};
+    *reinterpret_cast<uint2*>(p) = *reinterpret_cast<const uint2*>(h);
+  }
+}
+template <typename T>
+__device__ __forceinline__ float4 load4(const T* p) {
+  if constexpr (std::is_same<T, float>::value) {
+    return *reinterpret_cast<const float4*>(p);
+  } else {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    const T* h = reinterpret_cast<const T*>(&u);
+    return make_float4(to_f(h[0]), to_f(h[1]), to_f(h[2]), to_f(h[3]));
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(1024) k_norm_v(const float* __restrict__ x, const T* __restrict__ w,
+                                                 const T* __restrict__ b, float eps, int d, int layer_norm,
+                                                 T* __restrict__ out) {
+  __shared__ float red[32];
+  const int r = blockIdx.x, n4 = d >> 2, nt = blockDim.x;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
+  float4 v[4];
+  float sum = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int i = threadIdx.x + k * nt;
+    v[k] = i < n4 ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    sum += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+  }
+  const float mean = layer_norm ? block_sum(sum, red) / (float)d : 0.f;
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (threadIdx.x + k * nt < n4) {
+      const float a = v[k].x - mean, bb = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
+      ss += (a * a + bb * bb) + (c * c + e * e);
+    }
+  }
+  const float rstd = rsqrtf(block_sum(ss, red) / (float)d + eps);
+  T* orow = out + (size_t)r * d;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int i = threadIdx.x + k * nt;
+    if (i < n4) {
+      const float4 wv = load4(w + 4 * i);
+      float4 o = make_float4((v[k].x - mean) * rstd * wv.x, (v[k].y - mean) * rstd * wv.y,
+                             (v[k].z - mean) * rstd * wv.z, (v[k].w - mean) * rstd * wv.w);
+      if (layer_norm) {
+        const float4 bv = load4(b + 4 * i);
+        o.x += bv.x, o.y += bv.y, o.z += bv.z, o.w += bv.w;
+      }
+      store4(orow + 4 * i, o.x, o.y, o.z, o.w);
+    }
   }
 }
 
@@ -115,6 +181,63 @@ __global__ void k_rope_store(const float* __restrict__ qkv, const int* __restric
     const T v = f_to<T>(row[(Hq + Hkv) * dh + idx]);
     if (v_out) v_out[(size_t)r * Hkv * dh + idx] = v;
     if (pv) pv[(size_t)h * PAGE * dh + c] = v;
+  }
+}
+
+// Vectorised form for dh % 8 == 0: each thread rotates four consecutive pairs (i .. i+3, i+half ..
+// i+half+3) of one head with float4 loads and 4-element stores.
+template <typename T>
+__global__ void __launch_bounds__(256) k_rope_store_v(const float* __restrict__ qkv, const int* __restrict__ positions,
+                                                      const float2* __restrict__ rope, int Hq, int Hkv, int dh,
+                                                      T* __restrict__ q_out, T* __restrict__ k_out,
+                                                      T* __restrict__ v_out, KvSink sink) {
+  const int r = blockIdx.x;
+  const int pos = positions[r];
+  const int half = dh / 2, gph = half / 4;  // 4-pair groups per head
+  const float* row = qkv + (size_t)r * (Hq + 2 * Hkv) * dh;
+  T* pk = nullptr;
+  T* pv = nullptr;
+  if (sink.pool_layer) {
+    const int seq = sink.row_seq ? sink.row_seq[r] : 0;
+    const int page = sink.page_table[(size_t)seq * sink.pt_stride + pos / PAGE];
+    T* base = reinterpret_cast<T*>(sink.pool_layer) + (size_t)page * 2 * Hkv * PAGE * dh + (size_t)(pos % PAGE) * dh;
+    pk = base;
+    pv = base + (size_t)Hkv * PAGE * dh;
+  }
+  for (int idx = threadIdx.x; idx < (Hq + Hkv) * gph; idx += blockDim.x) {
+    const int h = idx / gph, i = (idx % gph) * 4;
+    const float* src = row + h * dh;
+    float4 y1 = *reinterpret_cast<const float4*>(src + i), y2 = *reinterpret_cast<const float4*>(src + i + half);
+    if (rope) {
+      const float4 c01 = *reinterpret_cast<const float4*>(rope + (size_t)pos * half + i);      // cos, sin of i, i+1
+      const float4 c23 = *reinterpret_cast<const float4*>(rope + (size_t)pos * half + i + 2);  // of i+2, i+3
+      const float4 x1 = y1, x2 = y2;
+      y1 = make_float4(x1.x * c01.x - x2.x * c01.y, x1.y * c01.z - x2.y * c01.w, x1.z * c23.x - x2.z * c23.y,
+                       x1.w * c23.z - x2.w * c23.w);
+      y2 = make_float4(x2.x * c01.x + x1.x * c01.y, x2.y * c01.z + x1.y * c01.w, x2.z * c23.x + x1.z * c23.y,
+                       x2.w * c23.z + x1.w * c23.w);
+    }
+    T* dsts[2] = {nullptr, nullptr};
+    if (h < Hq) {
+      dsts[0] = q_out + ((size_t)r * Hq + h) * dh;
+    } else {
+      const int kh = h - Hq;
+      if (k_out) dsts[0] = k_out + ((size_t)r * Hkv + kh) * dh;
+      if (pk) dsts[1] = pk + (size_t)kh * PAGE * dh;
+    }
+#pragma unroll
+    for (int t = 0; t < 2; ++t) {
+      if (!dsts[t]) continue;
+      store4(dsts[t] + i, y1.x, y1.y, y1.z, y1.w);
+      store4(dsts[t] + i + half, y2.x, y2.y, y2.z, y2.w);
+    }
+  }
+  const float* vrow = row + (Hq + Hkv) * dh;
+  for (int idx = threadIdx.x; idx < Hkv * dh / 4; idx += blockDim.x) {
+    const int h = (4 * idx) / dh, c = (4 * idx) % dh;
+    const float4 v = *reinterpret_cast<const float4*>(vrow + 4 * idx);
+    if (v_out) store4(v_out + (size_t)r * Hkv * dh + 4 * idx, v.x, v.y, v.z, v.w);
+    if (pv) store4(pv + (size_t)h * PAGE * dh + c, v.x, v.y, v.z, v.w);
   }
 }
 
@@ -206,7 +329,14 @@ sr_status launch_norm(int et, int norm, const float* x, const void* w, const voi
                       void* out, cudaStream_t st) {
   if (M == 0) return SR_OK;
   const int ln = norm == SR_NORM_LAYER;
-  SR_DISPATCH_ET(et, T, (k_norm<T><<<M, threads_for(d), 0, st>>>(x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
+  const bool aligned = ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(w) |
+                         reinterpret_cast<uintptr_t>(b) | reinterpret_cast<uintptr_t>(out)) & 15) == 0;
+  if (d % 4 == 0 && d <= 16 * 1024 && aligned) {
+    const int nt = std::max(32, ((d / 16 + 31) / 32) * 32);  // up to four float4 per thread
+    SR_DISPATCH_ET(et, T, (k_norm_v<T><<<M, nt, 0, st>>>(x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
+  } else {
+    SR_DISPATCH_ET(et, T, (k_norm<T><<<M, threads_for(d), 0, st>>>(x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
+  }
   SR_LAUNCH();
   return SR_OK;
 }
@@ -221,8 +351,16 @@ sr_status launch_rope_table(float2* tab, int max_pos, int head_dim, double theta
 sr_status launch_rope_store(int et, const float* qkv, int M, const int* positions, const float2* rope, int Hq,
                             int Hkv, int dh, void* q_out, void* k_out, void* v_out, KvSink sink, cudaStream_t st) {
   if (M == 0) return SR_OK;
-  SR_DISPATCH_ET(et, T, (k_rope_store<T><<<M, 128, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (T*)q_out, (T*)k_out,
-                                                            (T*)v_out, sink)));
+  const bool aligned = ((reinterpret_cast<uintptr_t>(qkv) | reinterpret_cast<uintptr_t>(rope) |
+                         reinterpret_cast<uintptr_t>(q_out) | reinterpret_cast<uintptr_t>(k_out) |
+                         reinterpret_cast<uintptr_t>(v_out) | reinterpret_cast<uintptr_t>(sink.pool_layer)) & 15) == 0;
+  if (dh % 8 == 0 && aligned) {
+    SR_DISPATCH_ET(et, T, (k_rope_store_v<T><<<M, 256, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (T*)q_out,
+                                                                (T*)k_out, (T*)v_out, sink)));
+  } else {
+    SR_DISPATCH_ET(et, T, (k_rope_store<T><<<M, 128, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (T*)q_out,
+                                                              (T*)k_out, (T*)v_out, sink)));
+  }
   SR_LAUNCH();
   return SR_OK;
 }
