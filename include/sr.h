@@ -121,14 +121,18 @@ typedef struct {
   int pool_pages;                         /* pages in the KV pool */
   int peak_pages_in_use;
   double ms_prefill, ms_decode, ms_score, ms_select, ms_total; /* wall-clock phases, stream-synchronised */
-  /* per kernel class (zero unless profiling is on): summed CUDA-event time of the launches on the
-     context's stream, launch count, and the algorithmic work of those launches -- 2 M N K flops for
-     a GEMM, 4 dh (keys) flops per query head for attention; bytes = operands read + results
-     written once (decode attention: the shared prompt KV once plus each candidate's own KV) */
-  double kern_ms[SR_KC_N];
-  long long kern_launches[SR_KC_N];
-  double kern_flops[SR_KC_N];
-  double kern_bytes[SR_KC_N];
+  /* per kernel class (zero unless profiling is on): launch count and algorithmic work of all
+     launches -- 2 M N K flops for a GEMM, 4 dh (keys) flops per query head for attention; bytes =
+     operands read + results written once (decode attention: the shared prompt KV once plus each
+     candidate's own KV) -- and, for the launches timed with CUDA events on the context's stream
+     (all of them, or one in `period`, see sr_set_profiling), their count, summed time and work */
+  double kern_ms[SR_KC_N];          /* summed event time of the timed launches */
+  long long kern_launches[SR_KC_N]; /* all launches */
+  double kern_flops[SR_KC_N];       /* all launches */
+  double kern_bytes[SR_KC_N];       /* all launches */
+  long long kern_timed[SR_KC_N];    /* timed launches */
+  double kern_timed_flops[SR_KC_N];
+  double kern_timed_bytes[SR_KC_N];
 } sr_stats;
 
 typedef struct sr_ctx sr_ctx;
@@ -156,7 +160,9 @@ void sr_destroy(sr_ctx* ctx);
 const char* sr_last_error(void);
 /* Use `stream` (a cudaStream_t) for all later work of this context; NULL restores the context's stream. */
 sr_status sr_set_stream(sr_ctx* ctx, void* stream);
-/* Turn per-kernel-class CUDA-event timing on (1) or off (0); results land in sr_stats.kern_*. */
+/* Per-kernel-class CUDA-event timing: 0 off; k >= 1 times one launch in k of each class (1: every
+   launch; each timed launch adds two event records to the stream) and counts all of them.  Results
+   land in sr_stats.kern_*.  Errors: SR_ERR_INVALID_ARG (null context, k < 0). */
 sr_status sr_set_profiling(sr_ctx* ctx, int enable);
 
 /*

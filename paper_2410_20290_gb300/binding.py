@@ -53,7 +53,9 @@ class sr_stats(ctypes.Structure):
                 ("peak_pages_in_use", ctypes.c_int), ("ms_prefill", ctypes.c_double), ("ms_decode", ctypes.c_double),
                 ("ms_score", ctypes.c_double), ("ms_select", ctypes.c_double), ("ms_total", ctypes.c_double),
                 ("kern_ms", ctypes.c_double * SR_KC_N), ("kern_launches", ctypes.c_longlong * SR_KC_N),
-                ("kern_flops", ctypes.c_double * SR_KC_N), ("kern_bytes", ctypes.c_double * SR_KC_N)]
+                ("kern_flops", ctypes.c_double * SR_KC_N), ("kern_bytes", ctypes.c_double * SR_KC_N),
+                ("kern_timed", ctypes.c_longlong * SR_KC_N), ("kern_timed_flops", ctypes.c_double * SR_KC_N),
+                ("kern_timed_bytes", ctypes.c_double * SR_KC_N)]
 
     def as_dict(self) -> dict:
         r = self.rounds
@@ -62,7 +64,9 @@ class sr_stats(ctypes.Structure):
         for f in ("b_per_round", "step_per_round", "k_per_round", "accepted_per_round", "r_cut_per_round"):
             out[f] = list(getattr(self, f))[:n]
         out["kernels"] = {KERNEL_CLASSES[k]: dict(ms=self.kern_ms[k], launches=self.kern_launches[k],
-                                                  flops=self.kern_flops[k], bytes=self.kern_bytes[k])
+                                                  flops=self.kern_flops[k], bytes=self.kern_bytes[k],
+                                                  timed=self.kern_timed[k], timed_flops=self.kern_timed_flops[k],
+                                                  timed_bytes=self.kern_timed_bytes[k])
                           for k in range(SR_KC_N)}
         return out
 
@@ -173,8 +177,9 @@ def sr_destroy(ctx):
     LIB.sr_destroy(ctx)
 
 
-def sr_set_profiling(ctx, enable: bool = True):
-    _check(LIB.sr_set_profiling(ctx, int(bool(enable))))
+def sr_set_profiling(ctx, period: int = 1):
+    """0 / False: off; k >= 1: time one launch in k of each kernel class (True = every launch)."""
+    _check(LIB.sr_set_profiling(ctx, int(period)))
 
 
 def sr_set_stream(ctx, stream=None):

@@ -31,6 +31,7 @@ __global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, co
                                                      const int* __restrict__ slot_ids, const int* __restrict__ lens,
                                                      int Hkv, float scale_log2, int window, int max_splits,
                                                      T* __restrict__ out, float* __restrict__ part) {
+  pdl_entry();
   constexpr int VE = 16 / sizeof(T);  // elements per 16-byte vector
   constexpr int TPT = DH / VE;        // threads per token
   constexpr int NG = 128 / TPT;       // token groups per CTA
@@ -140,6 +141,7 @@ __global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, co
 template <typename T, int DH>
 __global__ void k_decode_combine(const float* __restrict__ part, const int* __restrict__ lens, int Hq, int window,
                                  int max_splits, int t_min, int sbase, T* __restrict__ out) {
+  pdl_entry();
   const int hq = blockIdx.x, s = blockIdx.y, d = threadIdx.x;
   const int L = lens[s];
   const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
@@ -242,6 +244,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
                                                         const int* __restrict__ lens, int Hkv, float scale_log2,
                                                         int window, int t_min, int sbase, int max_splits,
                                                         T* __restrict__ out, float* __restrict__ part) {
+  pdl_entry();
   static_assert(G >= 1 && G <= 8 && DH % 16 == 0, "shape");
   constexpr int LDS = DH + 8;                  // padded smem row (elements): conflict-free ldmatrix
   constexpr int BLK = PAGE * LDS;              // one K or V page block in smem
@@ -460,6 +463,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
                                                       const int* __restrict__ tile_seq,
                                                       const int* __restrict__ tile_q0, int pos0, int Hq, int Hkv,
                                                       float scale_log2, int window, T* __restrict__ out) {
+  pdl_entry();
   constexpr int LD = DH + 8, LDV = DV + 8;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   T* sQ = reinterpret_cast<T*>(smem_raw);
@@ -616,6 +620,7 @@ __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, co
                                                      const int* __restrict__ lens, int n, int S, int Hkv,
                                                      float scale_log2, int window, int max_splits,
                                                      float* __restrict__ part) {
+  pdl_entry();
   constexpr int HPC = G < 4 ? G : 4;       // query heads per CTA
   constexpr int CPC = 4 / HPC;             // 16-candidate blocks per CTA
   constexpr int LD = DH + 8;
@@ -764,6 +769,7 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
                                    const float* __restrict__ vpre, int npre, const int* __restrict__ seq_off,
                                    int n_seq, int pos0, int Hq, int Hkv, int dh, float scale, int window,
                                    float* __restrict__ out) {
+  pdl_entry();
   extern __shared__ float sc[];
   __shared__ float red[32];
   const int r = blockIdx.x, hq = blockIdx.y, hk = hq / (Hq / Hkv);
@@ -824,7 +830,7 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
       SR_CUDA(cudaFuncSetAttribute(k_prefix_attn<T, DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem));
       pattr = true;
     }
-    k_prefix_attn<T, DH, G><<<dim3((b + 16 * CPC - 1) / (16 * CPC), Hkv * (G / HPC)), 128, psmem, st>>>(
+    launch_k(k_prefix_attn<T, DH, G>, dim3((b + 16 * CPC - 1) / (16 * CPC), Hkv * (G / HPC)), 128, psmem, st, 
         (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, b, shared_pos, Hkv,
         1.4426950408889634f / sqrtf((float)DH), window, max_splits, part);
     SR_LAUNCH();
@@ -839,11 +845,11 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid(Hkv, b, max_splits - sbase);
-  k_decode_attn_tc<T, DH, G><<<grid, 128, smem, st>>>((const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
+  launch_k(k_decode_attn_tc<T, DH, G>, grid, 128, smem, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
                                                        scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
   SR_LAUNCH();
   if (max_splits - sbase > 1) {  // some row has several position splits (a lone split merges the prefix itself)
-    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, t_min, sbase,
+    launch_k(k_decode_combine<T, DH>, dim3(Hkv * G, b), DH, 0, st, part, lens, Hkv * G, window, max_splits, t_min, sbase,
                                                              (T*)out);
     SR_LAUNCH();
   }
@@ -856,11 +862,11 @@ sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_s
                         cudaStream_t st) {
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid(Hkv, b, max_splits);
-  k_decode_attn<T, DH, G><<<grid, 128, 0, st>>>((const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
+  launch_k(k_decode_attn<T, DH, G>, grid, 128, 0, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
                                                  scale_log2, window, max_splits, (T*)out, part);
   SR_LAUNCH();
   if (max_splits > 1) {
-    k_decode_combine<T, DH><<<dim3(Hkv * G, b), DH, 0, st>>>(part, lens, Hkv * G, window, max_splits, 0, 0,
+    launch_k(k_decode_combine<T, DH>, dim3(Hkv * G, b), DH, 0, st, part, lens, Hkv * G, window, max_splits, 0, 0,
                                                              (T*)out);
     SR_LAUNCH();
   }
@@ -879,7 +885,7 @@ sr_status prefill_t(const void* q, const void* k, const void* v, const void* kpr
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid(n_tiles, Hq, DH / DV);
-  k_prefill_attn<T, DH, DV><<<grid, 128, smem, st>>>((const T*)q, (const T*)k, (const T*)v, (const T*)kpre,
+  launch_k(k_prefill_attn<T, DH, DV>, grid, 128, smem, st, (const T*)q, (const T*)k, (const T*)v, (const T*)kpre,
                                                       (const T*)vpre, npre, seq_off, tile_seq, tile_q0, pos0, Hq, Hkv,
                                                       scale_log2, window, (T*)out);
   SR_LAUNCH();
@@ -940,7 +946,7 @@ sr_status launch_prefill_attention_f32(const float* q, const float* k, const flo
     SR_CUDA(cudaFuncSetAttribute(k_prefill_attn_f32, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     attr = smem;
   }
-  k_prefill_attn_f32<<<dim3(rows, Hq), 128, smem, st>>>(q, k, v, kpre, vpre, npre, seq_off, n_seq, pos0, Hq, Hkv, dh,
+  launch_k(k_prefill_attn_f32, dim3(rows, Hq), 128, smem, st, q, k, v, kpre, vpre, npre, seq_off, n_seq, pos0, Hq, Hkv, dh,
                                                         1.f / sqrtf((float)dh), window, out);
   SR_LAUNCH();
   return SR_OK;

@@ -32,6 +32,35 @@ sr_status set_err(sr_status s, const char* fmt, ...);
                            __FILE__, __LINE__, #call, cudaGetErrorString(e_));                        \
   } while (0)
 #define SR_LAUNCH() SR_CUDA(cudaGetLastError())
+
+// Programmatic dependent launch: every kernel of the library starts with pdl_entry(), which waits until
+// the preceding kernel of the stream has completed and its writes are visible (a no-op when the kernel
+// was launched without the attribute) and then lets the next kernel's CTAs be scheduled, so launch
+// latency and prologues overlap the previous kernel's tail.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_entry() {
+  pdl_wait();
+  pdl_launch_next();
+}
+bool pdl_enabled();  // SR_PDL=0 in the environment turns the launch attribute off
+
+// Launch `k` on `st` with the programmatic-stream-serialisation attribute; errors surface through
+// cudaGetLastError (SR_LAUNCH).
+template <typename... KArgs, typename... Args>
+inline void launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  (void)cudaLaunchKernelEx(&cfg, k, static_cast<KArgs>(args)...);
+}
 #define SR_TRY(expr)               \
   do {                             \
     sr_status s_ = (expr);         \

@@ -16,6 +16,7 @@ namespace {
 template <typename T>
 __global__ void k_embed(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, const int* __restrict__ tokens,
                         const int* __restrict__ positions, int d, float* __restrict__ x) {
+  pdl_entry();
   const int r = blockIdx.x;
   const T* te = tok_emb + (size_t)tokens[r] * d;
   const T* pe = pos_emb ? pos_emb + (size_t)positions[r] * d : nullptr;
@@ -30,6 +31,7 @@ __global__ void k_embed(const T* __restrict__ tok_emb, const T* __restrict__ pos
 template <typename T>
 __global__ void k_norm(const float* __restrict__ x, const T* __restrict__ w, const T* __restrict__ b, float eps,
                        int d, int layer_norm, T* __restrict__ out) {
+  pdl_entry();
   __shared__ float red[32];
   const int r = blockIdx.x;
   const float* xr = x + (size_t)r * d;
@@ -79,6 +81,7 @@ template <typename T>
 __global__ void __launch_bounds__(1024) k_norm_v(const float* __restrict__ x, const T* __restrict__ w,
                                                  const T* __restrict__ b, float eps, int d, int layer_norm,
                                                  T* __restrict__ out) {
+  pdl_entry();
   __shared__ float red[32];
   const int r = blockIdx.x, n4 = d >> 2, nt = blockDim.x;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
@@ -119,6 +122,7 @@ __global__ void __launch_bounds__(1024) k_norm_v(const float* __restrict__ x, co
 
 // cos/sin of p * theta^(-2i/dh), evaluated in double precision and rounded once.
 __global__ void k_rope_table(float2* tab, int max_pos, int half, int dh, double theta) {
+  pdl_entry();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= max_pos * half) return;
   const int p = i / half, j = i % half;
@@ -133,6 +137,7 @@ template <typename T>
 __global__ void k_rope_store(const float* __restrict__ qkv, const int* __restrict__ positions,
                              const float2* __restrict__ rope, int Hq, int Hkv, int dh, T* __restrict__ q_out,
                              T* __restrict__ k_out, T* __restrict__ v_out, KvSink sink) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int pos = positions[r];
   const int half = dh / 2;
@@ -191,6 +196,7 @@ __global__ void __launch_bounds__(256) k_rope_store_v(const float* __restrict__ 
                                                       const float2* __restrict__ rope, int Hq, int Hkv, int dh,
                                                       T* __restrict__ q_out, T* __restrict__ k_out,
                                                       T* __restrict__ v_out, KvSink sink) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int pos = positions[r];
   const int half = dh / 2, gph = half / 4;  // 4-pair groups per head
@@ -249,6 +255,7 @@ __device__ __forceinline__ float gelu_d(float x) {
 // fp32 path: gated activations read gate/up interleaved in blocks of 32 columns.
 template <typename T>
 __global__ void k_act(const float* __restrict__ in, int F, int act, T* __restrict__ out) {
+  pdl_entry();
   const int r = blockIdx.x;
   for (int j = threadIdx.x; j < F; j += blockDim.x) {
     float v;
@@ -269,6 +276,7 @@ template <typename T>
 __global__ void k_score_head(const float* __restrict__ x, const int* __restrict__ rows, const T* __restrict__ w,
                              const T* __restrict__ b, float eps, int layer_norm, const T* __restrict__ head, int d,
                              float* __restrict__ rewards) {
+  pdl_entry();
   __shared__ float red[32];
   const float* xr = x + (size_t)rows[blockIdx.x] * d;
   float mean = 0.f;
@@ -296,6 +304,7 @@ __global__ void k_score_head(const float* __restrict__ x, const int* __restrict_
 // Copy page `src` to pages dst[0..n) in every layer (prompt-tail KV into each candidate's page).
 template <typename T>
 __global__ void k_copy_page(T* pool, long long layer_stride, int page_elems, int src, const int* __restrict__ dst) {
+  pdl_entry();
   const int l = blockIdx.y, j = blockIdx.x;
   const T* s = pool + (size_t)l * layer_stride + (size_t)src * page_elems;
   T* t = pool + (size_t)l * layer_stride + (size_t)dst[j] * page_elems;
@@ -305,6 +314,7 @@ __global__ void k_copy_page(T* pool, long long layer_stride, int page_elems, int
 // bf16 bit patterns -> fp16 bit patterns, in place (exact for |x| in [2^-17, 65504]; smaller
 // magnitudes round to the fp16 subnormal grid, larger ones saturate)
 __global__ void k_bf16_to_f16(uint16_t* p, size_t n) {
+  pdl_entry();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
     const float v = __uint_as_float((uint32_t)p[i] << 16);
     const f16 h = f_to<f16>(v);
@@ -319,7 +329,7 @@ int threads_for(int d) { return d >= 1024 ? 256 : (d >= 256 ? 128 : 64); }
 sr_status launch_embed(int et, const void* tok_emb, const void* pos_emb, const int* tokens, const int* positions,
                        int M, int d, float* x, cudaStream_t st) {
   if (M == 0) return SR_OK;
-  SR_DISPATCH_ET(et, T, (k_embed<T><<<M, threads_for(d), 0, st>>>((const T*)tok_emb, (const T*)pos_emb, tokens,
+  SR_DISPATCH_ET(et, T, (launch_k(k_embed<T>, M, threads_for(d), 0, st, (const T*)tok_emb, (const T*)pos_emb, tokens,
                                                                   positions, d, x)));
   SR_LAUNCH();
   return SR_OK;
@@ -333,9 +343,9 @@ sr_status launch_norm(int et, int norm, const float* x, const void* w, const voi
                          reinterpret_cast<uintptr_t>(b) | reinterpret_cast<uintptr_t>(out)) & 15) == 0;
   if (d % 4 == 0 && d <= 16 * 1024 && aligned) {
     const int nt = std::max(32, ((d / 16 + 31) / 32) * 32);  // up to four float4 per thread
-    SR_DISPATCH_ET(et, T, (k_norm_v<T><<<M, nt, 0, st>>>(x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
+    SR_DISPATCH_ET(et, T, (launch_k(k_norm_v<T>, M, nt, 0, st, x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
   } else {
-    SR_DISPATCH_ET(et, T, (k_norm<T><<<M, threads_for(d), 0, st>>>(x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
+    SR_DISPATCH_ET(et, T, (launch_k(k_norm<T>, M, threads_for(d), 0, st, x, (const T*)w, (const T*)b, eps, d, ln, (T*)out)));
   }
   SR_LAUNCH();
   return SR_OK;
@@ -343,7 +353,7 @@ sr_status launch_norm(int et, int norm, const float* x, const void* w, const voi
 
 sr_status launch_rope_table(float2* tab, int max_pos, int head_dim, double theta, cudaStream_t st) {
   const int n = max_pos * (head_dim / 2);
-  k_rope_table<<<(n + 255) / 256, 256, 0, st>>>(tab, max_pos, head_dim / 2, head_dim, theta);
+  launch_k(k_rope_table, (n + 255) / 256, 256, 0, st, tab, max_pos, head_dim / 2, head_dim, theta);
   SR_LAUNCH();
   return SR_OK;
 }
@@ -355,10 +365,10 @@ sr_status launch_rope_store(int et, const float* qkv, int M, const int* position
                          reinterpret_cast<uintptr_t>(q_out) | reinterpret_cast<uintptr_t>(k_out) |
                          reinterpret_cast<uintptr_t>(v_out) | reinterpret_cast<uintptr_t>(sink.pool_layer)) & 15) == 0;
   if (dh % 8 == 0 && aligned) {
-    SR_DISPATCH_ET(et, T, (k_rope_store_v<T><<<M, 256, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (T*)q_out,
+    SR_DISPATCH_ET(et, T, (launch_k(k_rope_store_v<T>, M, 256, 0, st, qkv, positions, rope, Hq, Hkv, dh, (T*)q_out,
                                                                 (T*)k_out, (T*)v_out, sink)));
   } else {
-    SR_DISPATCH_ET(et, T, (k_rope_store<T><<<M, 128, 0, st>>>(qkv, positions, rope, Hq, Hkv, dh, (T*)q_out,
+    SR_DISPATCH_ET(et, T, (launch_k(k_rope_store<T>, M, 128, 0, st, qkv, positions, rope, Hq, Hkv, dh, (T*)q_out,
                                                               (T*)k_out, (T*)v_out, sink)));
   }
   SR_LAUNCH();
@@ -367,7 +377,7 @@ sr_status launch_rope_store(int et, const float* qkv, int M, const int* position
 
 sr_status launch_act(int et, int act, const float* in, int M, int F, void* out, cudaStream_t st) {
   if (M == 0) return SR_OK;
-  SR_DISPATCH_ET(et, T, (k_act<T><<<M, 128, 0, st>>>(in, F, act, (T*)out)));
+  SR_DISPATCH_ET(et, T, (launch_k(k_act<T>, M, 128, 0, st, in, F, act, (T*)out)));
   SR_LAUNCH();
   return SR_OK;
 }
@@ -376,7 +386,7 @@ sr_status launch_score_head(int et, int norm, const float* x, const int* rows, i
                             float eps, const void* head, int d, float* rewards, cudaStream_t st) {
   if (n == 0) return SR_OK;
   const int ln = norm == SR_NORM_LAYER;
-  SR_DISPATCH_ET(et, T, (k_score_head<T><<<n, threads_for(d), 0, st>>>(x, rows, (const T*)w, (const T*)b, eps, ln,
+  SR_DISPATCH_ET(et, T, (launch_k(k_score_head<T>, n, threads_for(d), 0, st, x, rows, (const T*)w, (const T*)b, eps, ln,
                                                                        (const T*)head, d, rewards)));
   SR_LAUNCH();
   return SR_OK;
@@ -386,7 +396,7 @@ sr_status launch_copy_page(int et, void* pool, long long layer_stride, int n_lay
                            const int* dst, int n_dst, cudaStream_t st) {
   if (n_dst == 0) return SR_OK;
   dim3 grid(n_dst, n_layers);
-  SR_DISPATCH_ET(et, T, (k_copy_page<T><<<grid, 256, 0, st>>>((T*)pool, layer_stride, page_elems, src, dst)));
+  SR_DISPATCH_ET(et, T, (launch_k(k_copy_page<T>, grid, 256, 0, st, (T*)pool, layer_stride, page_elems, src, dst)));
   SR_LAUNCH();
   return SR_OK;
 }
@@ -394,7 +404,7 @@ sr_status launch_copy_page(int et, void* pool, long long layer_stride, int n_lay
 sr_status launch_bf16_to_f16(void* p, size_t n, cudaStream_t st) {
   if (n == 0) return SR_OK;
   const size_t blocks = std::min<size_t>((n + 255) / 256, 65535 * 8);
-  k_bf16_to_f16<<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<uint16_t*>(p), n);
+  launch_k(k_bf16_to_f16, (unsigned)blocks, 256, 0, st, reinterpret_cast<uint16_t*>(p), n);
   SR_LAUNCH();
   return SR_OK;
 }

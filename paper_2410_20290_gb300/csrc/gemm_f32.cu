@@ -12,6 +12,7 @@ constexpr int TM = 64, TN = 64, TK = 16;
 
 __global__ void __launch_bounds__(256) k_gemm_f32(const float* __restrict__ A, const float* __restrict__ W,
                                                   float* __restrict__ C, int M, int N, int K, int epi) {
+  pdl_entry();
   __shared__ float sA[TK][TM + 4];
   __shared__ float sW[TK][TN + 4];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
@@ -59,7 +60,7 @@ sr_status gemm_f32(const float* A, const float* W, float* C, int M, int N, int K
   if (epi != EPI_F32 && epi != EPI_ADD_F32 && epi != EPI_STORE)
     return set_err(SR_ERR_INVALID_ARG, "gemm_f32: epilogue %d not supported for fp32", epi);
   dim3 grid((N + TN - 1) / TN, (M + TM - 1) / TM);
-  k_gemm_f32<<<grid, 256, 0, st>>>(A, W, C, M, N, K, epi);
+  launch_k(k_gemm_f32, grid, 256, 0, st, A, W, C, M, N, K, epi);
   SR_LAUNCH();
   return SR_OK;
 }

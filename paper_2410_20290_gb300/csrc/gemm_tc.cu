@@ -378,6 +378,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   if (CL == 2) cluster_sync();  // the peer's barriers are initialised before anyone signals them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_entry();  // prologue done; the operands written by the previous kernel are visible from here
 
   if (warp == 0) {
     if (lane == 0) {
@@ -580,6 +581,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   cluster_sync();  // both CTAs' barriers are initialised (and TMEM allocated) before any cross-CTA signal
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_entry();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -765,15 +767,17 @@ sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs&
   const int groups_total = ((M + TM * CL - 1) / (TM * CL)) * ((N + BN - 1) / BN);
   const int groups = std::min(groups_total, max_groups);
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = CL, attr[0].val.clusterDim.y = 1, attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
   cfg.gridDim = dim3(groups * CL);
   cfg.blockDim = dim3(C::THREADS);
   cfg.dynamicSmemBytes = C::SMEM_BYTES;
   cfg.stream = st;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   SR_CUDA(cudaLaunchKernelEx(&cfg, k_gemm_tc<TM, BN, CL>, ta, tb, ep, M, N, K, g_err));
   return SR_OK;
 }
@@ -805,7 +809,7 @@ sr_status launch_pair(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArg
   }
   const int tiles = ((M + 255) / 256) * ((N + BNP - 1) / BNP);
   const int pairs = std::min(tiles, max_pairs);
-  k_gemm_pair<BNP><<<pairs * 2, C::THREADS, C::SMEM_BYTES, st>>>(ta, tb, ep, M, N, K, g_err);
+  launch_k(k_gemm_pair<BNP>, pairs * 2, C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err);
   SR_CUDA(cudaGetLastError());
   return SR_OK;
 }

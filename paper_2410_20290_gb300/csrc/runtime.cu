@@ -12,6 +12,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <cstdlib>
 #include <vector>
 
 #include "common.cuh"
@@ -31,6 +32,14 @@ sr_status set_err(sr_status s, const char* fmt, ...) {
 }
 
 int* gemm_error_word();
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("SR_PDL");
+    return !(e && e[0] == '0');
+  }();
+  return on;
+}
 
 namespace {
 
@@ -61,11 +70,13 @@ double now_ms() {
 }
 
 // -------------------------------------------------------------------------------------------------
-// per-kernel-class timing: CUDA events recorded on the launching stream around each launch,
-// read back after the stream synchronises
+// per-kernel-class timing: CUDA events recorded on the launching stream around one launch in
+// `period` of each class (chosen by a hash of the class's launch counter, so repeating launch patterns
+// are sampled evenly), read back after the stream synchronises; every launch's work is counted
 // -------------------------------------------------------------------------------------------------
 struct Prof {
   bool on = false;
+  int period = 1;
   std::vector<cudaEvent_t> ev;
   size_t used = 0;
   struct Rec {
@@ -74,8 +85,10 @@ struct Prof {
     double fl, by;
   };
   std::vector<Rec> recs;
-  double ms[SR_KC_N] = {}, fl[SR_KC_N] = {}, by[SR_KC_N] = {};
-  long long n[SR_KC_N] = {};
+  double ms[SR_KC_N] = {}, fl[SR_KC_N] = {}, by[SR_KC_N] = {};     // timed launches
+  double fl_all[SR_KC_N] = {}, by_all[SR_KC_N] = {};                 // every launch
+  long long n[SR_KC_N] = {}, n_all[SR_KC_N] = {};
+  unsigned cnt[SR_KC_N] = {};
 
   cudaEvent_t take() {
     if (used == ev.size()) {
@@ -85,13 +98,19 @@ struct Prof {
     }
     return ev[used++];
   }
-  long long begin(cudaStream_t st) {
+  long long begin(int cls, cudaStream_t st) {
     if (!on) return -1;
+    const unsigned h = (cnt[cls]++ * 2654435761u) >> 16;
+    if (period > 1 && h % (unsigned)period != 0) return -2;  // counted, not timed
     const size_t i = used;
     cudaEventRecord(take(), st);
     return (long long)i;
   }
   void end(long long i, int cls, cudaStream_t st, double f, double b) {
+    if (i == -1) return;
+    n_all[cls] += 1;
+    fl_all[cls] += f;
+    by_all[cls] += b;
     if (i < 0) return;
     const size_t j = used;
     cudaEventRecord(take(), st);
@@ -111,7 +130,7 @@ struct Prof {
   void reset() {
     recs.clear();
     used = 0;
-    for (int c = 0; c < SR_KC_N; ++c) ms[c] = fl[c] = by[c] = 0, n[c] = 0;
+    for (int c = 0; c < SR_KC_N; ++c) ms[c] = fl[c] = by[c] = fl_all[c] = by_all[c] = 0, n[c] = n_all[c] = 0, cnt[c] = 0;
   }
   ~Prof() {
     for (cudaEvent_t e : ev) cudaEventDestroy(e);
@@ -126,7 +145,7 @@ struct Scope {
   cudaStream_t st;
   double f, b;
   Scope(Prof* p_, int cls_, cudaStream_t st_, double f_ = 0, double b_ = 0)
-      : p(p_), i(p_ ? p_->begin(st_) : -1), cls(cls_), st(st_), f(f_), b(b_) {}
+      : p(p_), i(p_ ? p_->begin(cls_, st_) : -1), cls(cls_), st(st_), f(f_), b(b_) {}
   ~Scope() {
     if (p) p->end(i, cls, st, f, b);
   }
@@ -712,6 +731,7 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
 
 __global__ void k_gather_rows(const int* __restrict__ ids, const int* __restrict__ off, const int* __restrict__ tok,
                               int max_new, int P, int* tok_rows, int* pos_rows, int* last_row) {
+  pdl_entry();
   const int j = blockIdx.x;
   const int id = ids[j], r0 = off[j], n = off[j + 1] - off[j];
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
@@ -785,7 +805,7 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
     const int* dtq = dts + ch.n_tiles;
     {
       Scope sc(&c->prof, SR_KC_ELEMENTWISE, c->st);
-      k_gather_rows<<<ch.ns, 128, 0, c->st>>>(did, doff, c->tok, b.max_new, b.P, tok_rows, pos_rows, c->last_row);
+      launch_k(k_gather_rows, ch.ns, 128, 0, c->st, did, doff, c->tok, b.max_new, b.P, tok_rows, pos_rows, c->last_row);
     }
     if ((status = [&]() -> sr_status { SR_LAUNCH(); return SR_OK; }()) != SR_OK) break;
     PrefillPlan plan;
@@ -963,9 +983,12 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
   c->prof.harvest();
   for (int k = 0; k < SR_KC_N; ++k) {
     S.kern_ms[k] = c->prof.ms[k];
-    S.kern_launches[k] = c->prof.n[k];
-    S.kern_flops[k] = c->prof.fl[k];
-    S.kern_bytes[k] = c->prof.by[k];
+    S.kern_timed[k] = c->prof.n[k];
+    S.kern_timed_flops[k] = c->prof.fl[k];
+    S.kern_timed_bytes[k] = c->prof.by[k];
+    S.kern_launches[k] = c->prof.n_all[k];
+    S.kern_flops[k] = c->prof.fl_all[k];
+    S.kern_bytes[k] = c->prof.by_all[k];
   }
   S.best_id = c->h_ctrl[C_BEST];
   S.peak_pages_in_use = c->h_ctrl[C_PEAK];
@@ -1049,7 +1072,9 @@ void sr_destroy(sr_ctx* c) {
 
 sr_status sr_set_profiling(sr_ctx* c, int enable) {
   if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
+  if (enable < 0) return set_err(SR_ERR_INVALID_ARG, "profiling period must be >= 0");
   c->prof.on = enable != 0;
+  c->prof.period = enable > 0 ? enable : 1;
   c->prof.reset();
   return SR_OK;
 }

@@ -68,6 +68,7 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
                                                     uint32_t k0, uint32_t k1, float temperature, float eos_bias,
                                                     int eos_id, int* __restrict__ tokens_out, int* tok_hist,
                                                     int max_new, int* lens, int* status) {
+  pdl_entry();
   __shared__ float s_best[THREADS / 32];
   __shared__ int s_idx[THREADS / 32];
   const int r = blockIdx.x;
@@ -131,7 +132,7 @@ sr_status launch_sample(const float* logits, long long ld, int b, int V, const i
                         int max_new, int* lens, int* status, cudaStream_t st) {
   if (b == 0) return SR_OK;
   if (!(temperature > 0.f)) return set_err(SR_ERR_INVALID_ARG, "temperature must be > 0");
-  k_sample<<<b, THREADS, 0, st>>>(logits, ld, V, orig_ids, steps, (uint32_t)(seed & 0xFFFFFFFFu),
+  launch_k(k_sample, b, THREADS, 0, st, logits, ld, V, orig_ids, steps, (uint32_t)(seed & 0xFFFFFFFFu),
                                   (uint32_t)(seed >> 32), temperature, eos_bias, eos_id, tokens_out, tok_hist, max_new,
                                   lens, status);
   SR_LAUNCH();

@@ -36,6 +36,7 @@ __device__ void note_peak(int* ctrl) {
 }
 
 __global__ void k_pool_init(int* free_stack, int n_pages, int* ctrl) {
+  pdl_entry();
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_pages; i += gridDim.x * blockDim.x) free_stack[i] = i;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     for (int c = 0; c < C_N; ++c) ctrl[c] = 0;
@@ -48,6 +49,7 @@ __global__ void k_pool_init(int* free_stack, int n_pages, int* ctrl) {
 // the prompt tail until it is copied into each candidate's first private page.
 __global__ void k_prompt_pages(int* free_stack, int* ctrl, int n_sh, int has_tail, int template_page,
                                int* prompt_row) {
+  pdl_entry();
   if (threadIdx.x != 0) return;
   int top = ctrl[C_TOP];
   if (top < n_sh) {
@@ -66,6 +68,7 @@ __global__ void __launch_bounds__(CT) k_admit(int start, int count, int n_sh, in
                                               const int* __restrict__ prompt_row, int* pt, int max_pages, int* len,
                                               int* status, int* live, int* rset, const int* free_stack, int* ctrl,
                                               int* tail_dst) {
+  pdl_entry();
   const int top = ctrl[C_TOP];
   if (has_tail && top < count) {
     if (threadIdx.x == 0) ctrl[C_ERR] = E_POOL_EMPTY;
@@ -100,6 +103,7 @@ __global__ void __launch_bounds__(CT) k_step_begin(int P, const int* __restrict_
                                                    int* pt, int max_pages, const int* free_stack,
                                                    const int* __restrict__ tok, int max_new, int* tok_in,
                                                    int* pos_in, int* kv_len) {
+  pdl_entry();
   __shared__ int tmp[40];
   __shared__ int s_total;
   const int n = ctrl[C_NLIVE];
@@ -148,6 +152,7 @@ __global__ void __launch_bounds__(CT) k_step_begin(int P, const int* __restrict_
 // id, ascending page index) and leave the live list (stable compaction).
 __global__ void __launch_bounds__(CT) k_step_end(int P, int n_sh, int* live, int* ctrl, const int* len,
                                                  const int* status, const int* pt, int max_pages, int* free_stack) {
+  pdl_entry();
   __shared__ int tmp[40];
   __shared__ int s_rel, s_keep;
   const int n = ctrl[C_NLIVE];
@@ -228,6 +233,7 @@ __device__ __forceinline__ int cut_index(float alpha, int b) {
 
 __global__ void __launch_bounds__(CT) k_rcut(const float* __restrict__ rewards, int b, float alpha, int k_override,
                                              float* r_cut_out, uint8_t* mask_out) {
+  pdl_entry();
   __shared__ uint32_t keys[MAX_BATCH];
   __shared__ int hist[256];
   __shared__ int sh[4];
@@ -246,6 +252,7 @@ __global__ void __launch_bounds__(CT) k_round(int P, int n_sh, float alpha, int 
                                               const float* __restrict__ rewards, int* rset, int* live, int* ctrl,
                                               float* ctrlf, int* status, const int* len, float* reward_final,
                                               const int* pt, int max_pages, int* free_stack, uint8_t* mask_out) {
+  pdl_entry();
   __shared__ uint32_t keys[MAX_BATCH];
   __shared__ int hist[256];
   __shared__ int sh[4];
@@ -359,6 +366,7 @@ __global__ void __launch_bounds__(CT) k_round(int P, int n_sh, float alpha, int 
 
 // Final scores of completed candidates not yet scored: ids[j] -> DONE with r[j].
 __global__ void k_mark_done(const int* ids, const float* r, int n, int* status, float* reward_final) {
+  pdl_entry();
   for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < n; j += gridDim.x * blockDim.x) {
     status[ids[j]] = ST_DONE;
     reward_final[ids[j]] = r[j];
@@ -370,6 +378,7 @@ __global__ void k_mark_done(const int* ids, const float* r, int n, int* status, 
 __global__ void __launch_bounds__(CT) k_final(int N, const int* status, const float* reward_final, const int* tok,
                                               int max_new, const int* len, int* out_tokens, int* out_len,
                                               float* out_score, int* ctrl) {
+  pdl_entry();
   __shared__ unsigned long long best_s;
   if (threadIdx.x == 0) best_s = 0ull;
   __syncthreads();
@@ -404,20 +413,20 @@ __global__ void __launch_bounds__(CT) k_final(int N, const int* status, const fl
 
 // ---- launchers used by the runtime ----
 sr_status ctl_pool_init(int* free_stack, int n_pages, int* ctrl, cudaStream_t st) {
-  k_pool_init<<<(n_pages + 1023) / 1024 > 0 ? (n_pages + 1023) / 1024 : 1, 1024, 0, st>>>(free_stack, n_pages, ctrl);
+  launch_k(k_pool_init, (n_pages + 1023) / 1024 > 0 ? (n_pages + 1023) / 1024 : 1, 1024, 0, st, free_stack, n_pages, ctrl);
   SR_LAUNCH();
   return SR_OK;
 }
 sr_status ctl_prompt_pages(int* free_stack, int* ctrl, int n_sh, int has_tail, int template_page, int* prompt_row,
                            cudaStream_t st) {
-  k_prompt_pages<<<1, 32, 0, st>>>(free_stack, ctrl, n_sh, has_tail, template_page, prompt_row);
+  launch_k(k_prompt_pages, 1, 32, 0, st, free_stack, ctrl, n_sh, has_tail, template_page, prompt_row);
   SR_LAUNCH();
   return SR_OK;
 }
 sr_status ctl_admit(int start, int count, int n_sh, int has_tail, const int* prompt_row, int* pt, int max_pages,
                     int* len, int* status, int* live, int* rset, const int* free_stack, int* ctrl, int* tail_dst,
                     cudaStream_t st) {
-  k_admit<<<1, CT, 0, st>>>(start, count, n_sh, has_tail, prompt_row, pt, max_pages, len, status, live, rset,
+  launch_k(k_admit, 1, CT, 0, st, start, count, n_sh, has_tail, prompt_row, pt, max_pages, len, status, live, rset,
                             free_stack, ctrl, tail_dst);
   SR_LAUNCH();
   return SR_OK;
@@ -425,34 +434,34 @@ sr_status ctl_admit(int start, int count, int n_sh, int has_tail, const int* pro
 sr_status ctl_step_begin(int P, const int* live, int* ctrl, const int* len, int* pt, int max_pages,
                          const int* free_stack, const int* tok, int max_new, int* tok_in, int* pos_in, int* kv_len,
                          cudaStream_t st) {
-  k_step_begin<<<1, CT, 0, st>>>(P, live, ctrl, len, pt, max_pages, free_stack, tok, max_new, tok_in, pos_in,
+  launch_k(k_step_begin, 1, CT, 0, st, P, live, ctrl, len, pt, max_pages, free_stack, tok, max_new, tok_in, pos_in,
                                  kv_len);
   SR_LAUNCH();
   return SR_OK;
 }
 sr_status ctl_step_end(int P, int n_sh, int* live, int* ctrl, const int* len, const int* status, const int* pt,
                        int max_pages, int* free_stack, cudaStream_t st) {
-  k_step_end<<<1, CT, 0, st>>>(P, n_sh, live, ctrl, len, status, pt, max_pages, free_stack);
+  launch_k(k_step_end, 1, CT, 0, st, P, n_sh, live, ctrl, len, status, pt, max_pages, free_stack);
   SR_LAUNCH();
   return SR_OK;
 }
 sr_status ctl_round(int P, int n_sh, float alpha, int pool_need, const float* rewards, int* rset, int* live,
                     int* ctrl, float* ctrlf, int* status, const int* len, float* reward_final, const int* pt,
                     int max_pages, int* free_stack, uint8_t* mask_out, cudaStream_t st) {
-  k_round<<<1, CT, 0, st>>>(P, n_sh, alpha, pool_need, rewards, rset, live, ctrl, ctrlf, status, len, reward_final,
+  launch_k(k_round, 1, CT, 0, st, P, n_sh, alpha, pool_need, rewards, rset, live, ctrl, ctrlf, status, len, reward_final,
                             pt, max_pages, free_stack, mask_out);
   SR_LAUNCH();
   return SR_OK;
 }
 sr_status ctl_mark_done(const int* ids, const float* r, int n, int* status, float* reward_final, cudaStream_t st) {
   if (n == 0) return SR_OK;
-  k_mark_done<<<(n + 255) / 256, 256, 0, st>>>(ids, r, n, status, reward_final);
+  launch_k(k_mark_done, (n + 255) / 256, 256, 0, st, ids, r, n, status, reward_final);
   SR_LAUNCH();
   return SR_OK;
 }
 sr_status ctl_final(int N, const int* status, const float* reward_final, const int* tok, int max_new, const int* len,
                     int* out_tokens, int* out_len, float* out_score, int* ctrl, cudaStream_t st) {
-  k_final<<<1, CT, 0, st>>>(N, status, reward_final, tok, max_new, len, out_tokens, out_len, out_score, ctrl);
+  launch_k(k_final, 1, CT, 0, st, N, status, reward_final, tok, max_new, len, out_tokens, out_len, out_score, ctrl);
   SR_LAUNCH();
   return SR_OK;
 }
@@ -460,7 +469,7 @@ sr_status ctl_final(int N, const int* status, const float* reward_final, const i
 sr_status launch_rcut(const float* rewards, int b, float alpha, int k_override, float* r_cut_out, uint8_t* mask_out,
                       cudaStream_t st) {
   if (b <= 0 || b > MAX_BATCH) return set_err(SR_ERR_INVALID_ARG, "rcut: b must be in [1, %d]", MAX_BATCH);
-  k_rcut<<<1, CT, 0, st>>>(rewards, b, alpha, k_override, r_cut_out, mask_out);
+  launch_k(k_rcut, 1, CT, 0, st, rewards, b, alpha, k_override, r_cut_out, mask_out);
   SR_LAUNCH();
   return SR_OK;
 }
