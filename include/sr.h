@@ -251,7 +251,7 @@ sr_status sr_k_rcut(const float* rewards, int b, float alpha, int k_override, fl
  * tcgen05 tensor-core kernel, SR_DT_F32 the fp32 SIMT kernel.  A [M][K] (lda = K),
  * W [N][K], both of `dtype`.  epilogue: 0 store fp32 C [M][N]; 1 add into fp32
  * C [M][N]; 2 store C as `dtype`; 3 SwiGLU / 4 GeGLU on column pairs
- * interleaved in blocks of 32 (W rows 64j..64j+31 gate block j, 64j+32..64j+63
+ * interleaved in blocks of 16 (W rows 32j..32j+15 gate block j, 32j+16..32j+31
  * up block j) storing `dtype` C [M][N/2]; 5 tanh-GELU storing `dtype` C [M][N]
  * (3-5 16-bit only).  Needs K % 8 == 0, N % 32 == 0 (N % 64 for 3, 4). */
 sr_status sr_k_gemm(int dtype, const void* A, const void* W, void* C, int M, int N, int K, int epilogue,

@@ -252,7 +252,7 @@ __device__ __forceinline__ float gelu_d(float x) {
   return 0.5f * x * (1.f + tanhf(0.7978845608028654f * (x + 0.044715f * x * x * x)));
 }
 
-// fp32 path: gated activations read gate/up interleaved in blocks of 32 columns.
+// fp32 path: gated activations read gate/up interleaved in blocks of 16 columns.
 template <typename T>
 __global__ void k_act(const float* __restrict__ in, int F, int act, T* __restrict__ out) {
   pdl_entry();
@@ -263,8 +263,8 @@ __global__ void k_act(const float* __restrict__ in, int F, int act, T* __restric
       v = gelu_d(in[(size_t)r * F + j]);
     } else {
       const float* row = in + (size_t)r * 2 * F;
-      const int blk = j / 32, o = j % 32;
-      const float g = row[blk * 64 + o], u = row[blk * 64 + 32 + o];
+      const int blk = j / 16, o = j % 16;
+      const float g = row[blk * 32 + o], u = row[blk * 32 + 16 + o];
       v = (act == SR_ACT_SWIGLU ? silu_d(g) : gelu_d(g)) * u;
     }
     out[(size_t)r * F + j] = f_to<T>(v);

@@ -29,6 +29,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdlib>
+#include <map>
 #include <mutex>
 
 #include "common.cuh"
@@ -275,10 +276,11 @@ __device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int
   if (ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU) {
 #pragma unroll 1
     for (int c = 0; c < BNC; c += 64) {
+      // gate / up rows interleaved in blocks of 16: columns c..c+15 gate, c+16..c+31 up, c+32.. the next pair
       float g[32], u[32];
       tmem_ld16(tbase + c, g);
-      tmem_ld16(tbase + c + 16, g + 16);
-      tmem_ld16(tbase + c + 32, u);
+      tmem_ld16(tbase + c + 16, u);
+      tmem_ld16(tbase + c + 32, g + 16);
       tmem_ld16(tbase + c + 48, u + 16);
       if (row < M && col0 + c < N) {
 #pragma unroll
@@ -698,6 +700,279 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   }
 }
 
+// ---------------------------------------------------------------------------------------------
+// Skinny GEMM (M <= 512 rows, the decode batch after rejection): the product is computed transposed,
+// C^T = W A^T, on a CTA pair.  The M = 256 side of each cta_group::2 MMA is 256 rows of W (128 per SM)
+// and the N side is every row of A (MP = Nb * Np rows, padded, Nb MMAs of N = Np), so each SM stages
+// 128 rows of W and MP / 2 rows of A per K block: for 308 rows, 36 KB for 128 x 320 x 64 MACs (146 flop
+// per staged byte, against 51 useful for 128 x 128 tiles of a 3-tile-high M).  Few W tiles exist
+// (N / 256), so the K range is split into `s_split` slices to fill the SMs; with s_split > 1 every unit
+// writes its fp32 partial C^T tile to `part` [s][M][N] and k_splitk_reduce adds the slices in slice
+// order and applies the epilogue.  TMEM per SM: MP columns per accumulator (two when 2 MP <= 512).
+struct SkinnyGeo {
+  int Np, nb, MP, sub_bytes, stage_bytes, stages, nacc, tmem_cols, s_split, kps, n_tiles;
+};
+
+__device__ __forceinline__ void store_row_val(const EpiArgs& ep, int m, int n, float v) {
+  if (ep.kind == EPI_F32) {
+    reinterpret_cast<float*>(ep.out)[(size_t)m * ep.ldo + n] = v;
+  } else if (ep.kind == EPI_ADD_F32) {
+    reinterpret_cast<float*>(ep.out)[(size_t)m * ep.ldo + n] += v;
+  } else {
+    if (ep.kind == EPI_GELU) v = gelu_f(v);
+    uint16_t h;
+    if (ep.bf) {
+      const __nv_bfloat16 b = __float2bfloat16_rn(v);
+      h = *reinterpret_cast<const uint16_t*>(&b);
+    } else {
+      const __half b = __float2half_rn(fminf(fmaxf(v, -65504.f), 65504.f));
+      h = *reinterpret_cast<const uint16_t*>(&b);
+    }
+    reinterpret_cast<uint16_t*>(ep.out)[(size_t)m * ep.ldo + n] = h;
+  }
+}
+
+template <int NB>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
+    k_gemm_skinny(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmA, EpiArgs ep,
+                  float* __restrict__ part, SkinnyGeo geo, int M, int N, int K, int* err) {
+  constexpr int MAXST = 8;
+  const int STAGES = geo.stages, STAGE_BYTES = geo.stage_bytes, SUB = geo.sub_bytes, Np = geo.Np, MP = geo.MP;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + PairCfg<256>::GUARD);
+  uint64_t* empty = full + MAXST;
+  uint64_t* tfull = empty + MAXST;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const uint32_t idesc = idesc_pair(ep.bf != 0, Np);
+  const int num_k = (K + BK - 1) / BK;
+  const int units = geo.n_tiles * geo.s_split;
+  const int t0 = blockIdx.x / 2, tstep = gridDim.x / 2;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 8);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(geo.tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_entry();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer: 128 W rows + this CTA's halves of the A blocks ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int armed[MAXST];
+      uint32_t armed_par[MAXST];
+      for (int s = 0; s < MAXST; ++s) armed[s] = 0, armed_par[s] = 0;
+      bool ok = true;
+      for (int u = t0; u < units && ok; u += tstep) {
+        const int tile = u % geo.n_tiles, slice = u / geo.n_tiles;
+        const int kb0 = slice * geo.kps, kb1 = min(num_k, kb0 + geo.kps);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (rank == 0) mbar_expect_tx(&full[stage], 2 * STAGE_BYTES);
+          const uint32_t bar = cluster_addr(&full[stage], 0);
+          uint8_t* st = smem + stage * STAGE_BYTES;
+          tma_load_2d_pair(st, &tmW, bar, kb * BK, tile * 256 + (int)rank * BM);
+#pragma unroll
+          for (int i = 0; i < NB; ++i)
+            tma_load_2d_pair(st + 16384 + i * SUB, &tmA, bar, kb * BK, i * Np + (int)rank * (Np / 2));
+          armed[stage] = 1;
+          armed_par[stage] = phase;
+          if (++stage == STAGES) stage = 0, phase ^= 1u;
+        }
+      }
+      if (!ok) {
+        atomicExch(err, 1);
+        *abort_flag = 1;
+        if (rank == 0) {
+          for (int s = 0; s < STAGES; ++s)
+            if (armed[s]) mbar_wait(&full[s], armed_par[s], nullptr);
+        } else {
+          const unsigned long long t = gtimer();
+          while (gtimer() - t < 1000000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---------------- MMA issuer (even CTA) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int u = t0; u < units && ok; u += tstep) {
+        const int slice = u / geo.n_tiles;
+        const int kb0 = slice * geo.kps, kb1 = min(num_k, kb0 + geo.kps);
+        if (!mbar_wait_cl(&tempty[acc], acc_phase ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * MP);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(smem + stage * STAGE_BYTES);
+          const uint64_t aw = sdesc(st);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+#pragma unroll
+            for (int i = 0; i < NB; ++i)
+              umma_pair(d_tmem + (uint32_t)(i * Np), aw + (uint64_t)(kk * 2),
+                        sdesc(st + 16384 + i * SUB) + (uint64_t)(kk * 2), idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+          }
+          umma_pair_commit_mc(&empty[stage], 0x3);
+          if (++stage == STAGES) stage = 0, phase ^= 1u;
+        }
+        if (!ok) break;
+        umma_pair_commit_mc(&tfull[acc], 0x3);
+        if (++acc == geo.nacc) acc = 0, acc_phase ^= 1u;
+      }
+      if (!ok) {
+        atomicExch(err, 2);
+        *abort_flag = 1;
+      }
+      umma_pair_commit_mc(mma_done, 0x1);
+      mbar_wait(mma_done, 0, nullptr);
+    }
+  } else {
+    // ---------------- epilogue: lane = one W row (output column n), TMEM column = output row m ----------
+    const int quad = warp & 3;
+    const bool gated = ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int u = t0; u < units; u += tstep) {
+      const int tile = u % geo.n_tiles, slice = u / geo.n_tiles;
+      int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag) : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          atomicExch(err, 3);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const int nbase = tile * 256 + (int)rank * BM + quad * 32;  // first W row of this warp (multiple of 32)
+      const int n = nbase + lane;
+      const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * MP);
+#pragma unroll 1
+      for (int c = 0; c < MP; c += 16) {
+        float v[16];
+        tmem_ld16(tbase + c, v);
+        if (c >= M || nbase >= N) continue;
+        if (geo.s_split > 1) {
+          float* dst = part + ((size_t)slice * M) * N + n;
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c + j < M) dst[(size_t)(c + j) * N] = v[j];
+        } else if (gated) {
+          // W rows interleave gate / up in blocks of 16: lanes 0-15 gate, 16-31 up of features 16 (nbase/32) + lane
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float up = __shfl_xor_sync(0xffffffffu, v[j], 16);
+            if (lane < 16 && c + j < M) {
+              const float a = ep.kind == EPI_SWIGLU ? silu_f(v[j]) : gelu_f(v[j]);
+              EpiArgs e2 = ep;
+              e2.kind = EPI_STORE;
+              store_row_val(e2, c + j, 16 * (nbase / 32) + lane, a * up);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c + j < M) store_row_val(ep, c + j, n, v[j]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cta(&tempty[acc], 0);
+      if (++acc == geo.nacc) acc = 0, acc_phase ^= 1u;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(geo.tmem_cols)
+                 : "memory");
+  }
+}
+
+// Sums the s fp32 partials of a split-K skinny GEMM in slice order and applies the epilogue.
+// Non-gated: one thread per 4 consecutive outputs of a row; gated: per 4 consecutive features.
+__global__ void __launch_bounds__(256) k_splitk_reduce(const float* __restrict__ part, int s, int M, int N,
+                                                       EpiArgs ep) {
+  pdl_entry();
+  const bool gated = ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU;
+  const int cols = gated ? N / 2 : N;
+  const size_t total = (size_t)M * (cols / 4);
+  for (size_t t = blockIdx.x * (size_t)blockDim.x + threadIdx.x; t < total; t += (size_t)gridDim.x * blockDim.x) {
+    const int m = (int)(t / (cols / 4)), c = (int)(t % (cols / 4)) * 4;
+    if (!gated) {
+      float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k = 0; k < s; ++k) {
+        const float4 p = *reinterpret_cast<const float4*>(part + ((size_t)k * M + m) * N + c);
+        a.x += p.x, a.y += p.y, a.z += p.z, a.w += p.w;
+      }
+      const float v[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) store_row_val(ep, m, c + j, v[j]);
+    } else {
+      const int ng = 32 * (c / 16) + c % 16;  // gate rows of features c..c+3; up rows 16 further
+      float4 g = make_float4(0.f, 0.f, 0.f, 0.f), u = g;
+      for (int k = 0; k < s; ++k) {
+        const float* row = part + ((size_t)k * M + m) * N;
+        const float4 pg = *reinterpret_cast<const float4*>(row + ng), pu = *reinterpret_cast<const float4*>(row + ng + 16);
+        g.x += pg.x, g.y += pg.y, g.z += pg.z, g.w += pg.w;
+        u.x += pu.x, u.y += pu.y, u.z += pu.z, u.w += pu.w;
+      }
+      const float gv[4] = {g.x, g.y, g.z, g.w}, uv[4] = {u.x, u.y, u.z, u.w};
+      EpiArgs e2 = ep;
+      e2.kind = EPI_STORE;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        store_row_val(e2, m, c + j, (ep.kind == EPI_SWIGLU ? silu_f(gv[j]) : gelu_f(gv[j])) * uv[j]);
+    }
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 int g_num_sms = 0;
@@ -705,6 +980,9 @@ int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
 int g_cl_override = 0;  // SR_GEMM_CL: force the cluster size (1 or 2)
 int g_tm_override = 0;  // SR_GEMM_TM: force the tile height (128 or 256)
 int g_pair_override = -1;  // SR_GEMM_PAIR: 1 forces the CTA-pair kernel, 0 forbids it
+int g_skinny_override = -1;  // SR_GEMM_SKINNY: 0 forbids the skinny kernel (else used for M <= 512)
+std::mutex g_ws_mu;
+std::map<int, std::pair<float*, size_t>> g_ws;  // per device: split-K partial workspace (floats)
 int* g_err = nullptr;
 
 // Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost.  The per-tile
@@ -814,6 +1092,106 @@ sr_status launch_pair(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArg
   return SR_OK;
 }
 
+sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, int K, int box_rows);
+
+sr_status skinny_workspace(size_t floats, float** out) {
+  int dev;
+  SR_CUDA(cudaGetDevice(&dev));
+  std::lock_guard<std::mutex> lk(g_ws_mu);
+  auto& w = g_ws[dev];
+  if (w.second < floats) {
+    if (w.first) SR_CUDA(cudaFree(w.first));
+    w.first = nullptr;
+    w.second = 0;
+    SR_CUDA(cudaMalloc(&w.first, floats * sizeof(float)));
+    w.second = floats;
+  }
+  *out = w.first;
+  return SR_OK;
+}
+
+constexpr int SKINNY_SMEM_MAX = 1024 + 192 * 1024 + PairCfg<256>::GUARD + BAR_BYTES;
+
+template <int NB>
+int skinny_max_pairs() {
+  static int max_pairs = 0;
+  if (!max_pairs) {
+    cudaFuncSetAttribute(k_gemm_skinny<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, SKINNY_SMEM_MAX);
+    max_pairs = g_num_sms / 2;
+    cudaLaunchConfig_t qc = {};
+    qc.gridDim = dim3(max_pairs * 2);
+    qc.blockDim = dim3(192);
+    qc.dynamicSmemBytes = SKINNY_SMEM_MAX;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, k_gemm_skinny<NB>, &qc) == cudaSuccess && clusters > 0)
+      max_pairs = std::min(max_pairs, clusters);
+    cudaGetLastError();
+  }
+  return max_pairs;
+}
+
+// Geometry and split of the skinny kernel for an M-row product (M <= 512).
+SkinnyGeo skinny_geometry(int M, int N, int K, int max_pairs) {
+  SkinnyGeo g{};
+  const int mp32 = (M + 31) / 32 * 32;
+  g.nb = mp32 > 256 ? 2 : 1;
+  g.Np = (mp32 / g.nb + 15) / 16 * 16;
+  g.MP = g.nb * g.Np;
+  g.sub_bytes = (g.Np / 2) * 128;
+  g.stage_bytes = 16384 + g.nb * g.sub_bytes;
+  g.stages = std::min(8, (192 * 1024) / g.stage_bytes);
+  g.nacc = 2 * g.MP <= 512 ? 2 : 1;
+  int cols = 32;
+  while (cols < g.nacc * g.MP) cols *= 2;
+  g.tmem_cols = cols;
+  g.n_tiles = (N + 255) / 256;
+  const int num_k = (K + BK - 1) / BK;
+  int s = g.n_tiles >= max_pairs ? 1 : std::max(1, max_pairs / g.n_tiles);
+  s = std::max(1, std::min({s, 8, num_k / 4}));
+  g.kps = (num_k + s - 1) / s;
+  g.s_split = (num_k + g.kps - 1) / g.kps;
+  return g;
+}
+
+// Where the skinny kernel measured faster on GB300 than the 128-row tiles: shapes with few W tiles,
+// where split-K fills the SMs (N below 256 x the SM pairs), and among those the narrow outputs
+// (N <= 4096: O and down projections), the large reductions (K >= 8192) and the small batches
+// (M <= 256).  Wide single-slice shapes (gate/up, LM head) stay on the one-SM tiles.
+bool pick_skinny(int M, int N, int K) {
+  if (M > 512) return false;
+  const int max_pairs = std::min(skinny_max_pairs<1>(), skinny_max_pairs<2>());
+  const SkinnyGeo g = skinny_geometry(M, N, K, max_pairs);
+  if (g.s_split < 2) return false;
+  return M <= 256 || K >= 8192 || N <= 4096;
+}
+
+sr_status launch_skinny(const void* A, const void* W, bool bf, const EpiArgs& ep, int M, int N, int K,
+                        cudaStream_t st) {
+  const int max_pairs = std::min(skinny_max_pairs<1>(), skinny_max_pairs<2>());
+  const SkinnyGeo g = skinny_geometry(M, N, K, max_pairs);
+  CUtensorMap tw, ta;
+  SR_TRY(encode_kmajor(&tw, W, bf, N, K, BM));
+  SR_TRY(encode_kmajor(&ta, A, bf, M, K, g.Np / 2));
+  float* part = nullptr;
+  if (g.s_split > 1) SR_TRY(skinny_workspace((size_t)g.s_split * M * N, &part));
+  const int units = g.n_tiles * g.s_split;
+  const int pairs = std::min(units, max_pairs);
+  const size_t smem = 1024 + (size_t)g.stages * g.stage_bytes + PairCfg<256>::GUARD + BAR_BYTES;
+  if (g.nb == 1)
+    launch_k(k_gemm_skinny<1>, pairs * 2, 192, smem, st, tw, ta, ep, part, g, M, N, K, g_err);
+  else
+    launch_k(k_gemm_skinny<2>, pairs * 2, 192, smem, st, tw, ta, ep, part, g, M, N, K, g_err);
+  SR_CUDA(cudaGetLastError());
+  if (g.s_split > 1) {
+    const bool gated = ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU;
+    const size_t total = (size_t)M * ((gated ? N / 2 : N) / 4);
+    const int blocks = (int)std::min<size_t>((total + 255) / 256, (size_t)g_num_sms * 8);
+    launch_k(k_splitk_reduce, blocks, 256, 0, st, (const float*)part, g.s_split, M, N, ep);
+    SR_CUDA(cudaGetLastError());
+  }
+  return SR_OK;
+}
+
 sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, int K, int box_rows) {
   std::call_once(g_encode_once, [] {
     void* fn = nullptr;
@@ -856,10 +1234,14 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     if (const char* e = getenv("SR_GEMM_CL")) g_cl_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_TM")) g_tm_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_PAIR")) g_pair_override = atoi(e);
+    if (const char* e = getenv("SR_GEMM_SKINNY")) g_skinny_override = atoi(e);
   }
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
   CUtensorMap ta, tb;
   EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
+  const bool forced = g_pair_override == 1 || g_bn_override != 0 || g_tm_override != 0 || g_cl_override != 0;
+  if (M <= 512 && g_skinny_override != 0 && (g_skinny_override == 1 || (!forced && pick_skinny(M, N, K))))
+    return launch_skinny(A, W, bf, ep, M, N, K, st);
   if (g_pair_override == 1 || (g_pair_override == -1 && g_bn_override == 0 && g_tm_override == 0 &&
                                g_cl_override == 0 && pick_pair(M, N, K, gated))) {
     SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));

@@ -196,7 +196,7 @@ sr_status check_desc(const sr_model_desc* m, const char* who) {
 }
 
 // Copy one model's blob (host or device; densely packed in the sr.h order) into an aligned
-// device allocation; gate/up rows are interleaved in blocks of 32 for the fused GLU epilogue.
+// device allocation; gate/up rows are interleaved in blocks of 16 for the fused GLU epilogues.
 sr_status load_model(Model& M, const sr_model_desc* d, const void* src) {
   M.d = *d;
   M.esz = d->dtype == SR_DT_F32 ? 4 : 2;
@@ -254,10 +254,10 @@ sr_status load_model(Model& M, const sr_model_desc* d, const void* src) {
     if (ts[i].kind == 0) {
       SR_CUDA(cudaMemcpy(dst, s + soff, bytes, cudaMemcpyDefault));
     } else {
-      // rows of block j (32 rows of D) land at rows 64j (gate) or 64j + 32 (up)
+      // rows of block j (16 rows of D) land at rows 32j (gate) or 32j + 16 (up)
       const size_t row_bytes = D * E;
-      char* base = dst + (ts[i].kind == 2 ? 32 * row_bytes : 0);
-      SR_CUDA(cudaMemcpy2D(base, 64 * row_bytes, s + soff, 32 * row_bytes, 32 * row_bytes, F / 32,
+      char* base = dst + (ts[i].kind == 2 ? 16 * row_bytes : 0);
+      SR_CUDA(cudaMemcpy2D(base, 32 * row_bytes, s + soff, 16 * row_bytes, 16 * row_bytes, F / 16,
                            cudaMemcpyDefault));
     }
     soff += bytes;

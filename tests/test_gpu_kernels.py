@@ -129,7 +129,7 @@ def test_gemm_tc_epilogues(sr, dt, epi, M, N, K):
     W = torch.randn(N, K, generator=g).to(T16[dt])
     acc = A.float() @ W.float().T
     if epi in (3, 4):
-        blk = acc.reshape(M, N // 64, 2, 32)
+        blk = acc.reshape(M, N // 32, 2, 16)
         gate, up = blk[:, :, 0, :].reshape(M, N // 2), blk[:, :, 1, :].reshape(M, N // 2)
         act = torch.nn.functional.silu(gate) if epi == 3 else torch.nn.functional.gelu(gate, approximate="tanh")
         ref = act * up
