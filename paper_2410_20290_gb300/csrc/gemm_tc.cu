@@ -31,6 +31,7 @@
 #include <cstdlib>
 #include <map>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -172,6 +173,19 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 lanes x 64 consecutive fp32 columns in one load and one wait.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + __expf(-x)); }
 __device__ __forceinline__ float gelu_f(float x) {
   const float c = 0.7978845608028654f;
@@ -277,42 +291,48 @@ __device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int
 #pragma unroll 1
     for (int c = 0; c < BNC; c += 64) {
       // gate / up rows interleaved in blocks of 16: columns c..c+15 gate, c+16..c+31 up, c+32.. the next pair
-      float g[32], u[32];
-      tmem_ld16(tbase + c, g);
-      tmem_ld16(tbase + c + 16, u);
-      tmem_ld16(tbase + c + 32, g + 16);
-      tmem_ld16(tbase + c + 48, u + 16);
+      float v[64];
+      tmem_ld64(tbase + c, v);
       if (row < M && col0 + c < N) {
+        float g[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) g[j] = (ep.kind == EPI_SWIGLU ? silu_f(g[j]) : gelu_f(g[j])) * u[j];
+        for (int j = 0; j < 32; ++j) {
+          const int gi = (j < 16) ? j : j + 16;
+          g[j] = (ep.kind == EPI_SWIGLU ? silu_f(v[gi]) : gelu_f(v[gi])) * v[gi + 16];
+        }
         uint16_t* dst = reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + (col0 + c) / 2;
         store16x32(dst, g, ep.bf != 0);
       }
     }
   } else {
 #pragma unroll 1
-    for (int c = 0; c < BNC; c += 32) {
-      float v[32];
-      tmem_ld16(tbase + c, v);
-      tmem_ld16(tbase + c + 16, v + 16);
-      if (row < M && col0 + c < N) {
-        if (ep.kind == EPI_F32 || ep.kind == EPI_ADD_F32) {
-          float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)row * ep.ldo + col0 + c);
+    for (int c = 0; c < BNC; c += 64) {
+      float v[64];
+      tmem_ld64(tbase + c, v);
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            if (ep.kind == EPI_ADD_F32) {
-              const float4 r = dst[q];
-              o.x += r.x, o.y += r.y, o.z += r.z, o.w += r.w;
+      for (int hh = 0; hh < 2; ++hh) {
+        float* w = v + 32 * hh;
+        const int cc = c + 32 * hh;
+        if (row < M && col0 + cc < N) {
+          if (ep.kind == EPI_F32 || ep.kind == EPI_ADD_F32) {
+            float4* dst =
+                reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)row * ep.ldo + col0 + cc);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              float4 o = make_float4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+              if (ep.kind == EPI_ADD_F32) {
+                const float4 r = dst[q];
+                o.x += r.x, o.y += r.y, o.z += r.z, o.w += r.w;
+              }
+              dst[q] = o;
             }
-            dst[q] = o;
-          }
-        } else {
-          if (ep.kind == EPI_GELU) {
+          } else {
+            if (ep.kind == EPI_GELU) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
+              for (int j = 0; j < 32; ++j) w[j] = gelu_f(w[j]);
+            }
+            store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col0 + cc, w, ep.bf != 0);
           }
-          store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col0 + c, v, ep.bf != 0);
         }
       }
     }
@@ -891,33 +911,50 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       const int nbase = tile * 256 + (int)rank * BM + quad * 32;  // first W row of this warp (multiple of 32)
       const int n = nbase + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * MP);
-#pragma unroll 1
-      for (int c = 0; c < MP; c += 16) {
-        float v[16];
-        tmem_ld16(tbase + c, v);
-        if (c >= M || nbase >= N) continue;
+      // one output column n per lane; TMEM column c = output row m
+      auto emit = [&](int c, const float* v, auto cnt_c) {
+        constexpr int cnt = decltype(cnt_c)::value;
         if (geo.s_split > 1) {
           float* dst = part + ((size_t)slice * M) * N + n;
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
+          for (int j = 0; j < cnt; ++j)
             if (c + j < M) dst[(size_t)(c + j) * N] = v[j];
         } else if (gated) {
           // W rows interleave gate / up in blocks of 16: lanes 0-15 gate, 16-31 up of features 16 (nbase/32) + lane
+          const int f = 16 * (nbase / 32) + lane;
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
+          for (int j = 0; j < cnt; ++j) {
             const float up = __shfl_xor_sync(0xffffffffu, v[j], 16);
             if (lane < 16 && c + j < M) {
-              const float a = ep.kind == EPI_SWIGLU ? silu_f(v[j]) : gelu_f(v[j]);
-              EpiArgs e2 = ep;
-              e2.kind = EPI_STORE;
-              store_row_val(e2, c + j, 16 * (nbase / 32) + lane, a * up);
+              const float a = (ep.kind == EPI_SWIGLU ? silu_f(v[j]) : gelu_f(v[j])) * up;
+              uint16_t* o = reinterpret_cast<uint16_t*>(ep.out) + (size_t)(c + j) * ep.ldo + f;
+              if (ep.bf) {
+                const __nv_bfloat16 b = __float2bfloat16_rn(a);
+                *o = *reinterpret_cast<const uint16_t*>(&b);
+              } else {
+                const __half b = __float2half_rn(fminf(fmaxf(a, -65504.f), 65504.f));
+                *o = *reinterpret_cast<const uint16_t*>(&b);
+              }
             }
           }
         } else {
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
+          for (int j = 0; j < cnt; ++j)
             if (c + j < M) store_row_val(ep, c + j, n, v[j]);
         }
+      };
+      int c = 0;
+#pragma unroll 1
+      for (; c + 64 <= MP; c += 64) {  // 64 columns per load / wait
+        float v[64];
+        tmem_ld64(tbase + c, v);
+        if (c < M && nbase < N) emit(c, v, std::integral_constant<int, 64>{});
+      }
+#pragma unroll 1
+      for (; c < MP; c += 16) {
+        float v[16];
+        tmem_ld16(tbase + c, v);
+        if (c < M && nbase < N) emit(c, v, std::integral_constant<int, 16>{});
       }
       tc_fence_before();
       __syncwarp();
