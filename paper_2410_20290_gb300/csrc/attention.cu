@@ -237,7 +237,10 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
 // the G real heads plus zero padding), the online softmax runs per head column across the 8 lanes
 // holding its 16 positions, and O^T += V^T P^T adds dh/16 tiles with P carried as an fp16/bf16
 // hi + lo pair.  Warps merge their (m, l, O) through shared memory at the end.
-template <typename T, int DH, int G>
+// WPH = 1 (short suffixes): the CTA's four warps take four kv heads of the slot instead, each warp walks
+// all pages of its head and writes its result itself -- a quarter of the CTAs, for suffixes of a few pages
+// where one CTA per (head, slot) would be mostly launch and merge latency.
+template <typename T, int DH, int G, int WPH>
 __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q, const T* __restrict__ pool,
                                                         const int* __restrict__ pt, int pt_stride,
                                                         const int* __restrict__ slot_ids,
@@ -257,7 +260,12 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
   uint16_t* sPh = reinterpret_cast<uint16_t*>(wbase + 4 * BLK);
   uint16_t* sPl = sPh + 8 * PAGE;
 
-  const int h = blockIdx.x, s = blockIdx.y, split = blockIdx.z;
+  static_assert(WPH == 4 || WPH == 1, "warps per head");
+  const int h_raw = WPH == 4 ? (int)blockIdx.x : (int)blockIdx.x * 4 + warp;
+  const bool hvalid = h_raw < Hkv;
+  const int h = hvalid ? h_raw : 0;
+  const int s = blockIdx.y, split = blockIdx.z;
+  const int pw = WPH == 4 ? warp : 0;  // this warp's first page of the split; pages step by WPH
   const int Hq = Hkv * G;
   const int L = lens[s];
   const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
@@ -265,7 +273,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
   if (split >= nsplit) return;
   const int t_begin = t_lo + split * SPLIT, t_end = min(L, t_begin + SPLIT);
   const int p_first = t_begin / PAGE, n_pages = (t_end - 1) / PAGE - p_first + 1;
-  const int my_pages = n_pages > warp ? (n_pages - warp + 3) / 4 : 0;
+  const int my_pages = (hvalid && n_pages > pw) ? (n_pages - pw + WPH - 1) / WPH : 0;
   const int* ptrow = pt + (size_t)slot_ids[s] * pt_stride;
   const size_t page_elems = (size_t)2 * Hkv * PAGE * DH;
   const size_t v_off = (size_t)Hkv * PAGE * DH;
@@ -281,7 +289,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
     }
   }
   auto issue = [&](int i, int stage) {
-    const int page = ptrow[p_first + warp + 4 * i];
+    const int page = ptrow[p_first + pw + WPH * i];
     const T* srcK = pool + (size_t)page * page_elems + (size_t)h * PAGE * DH;
     const T* srcV = srcK + v_off;
     T* dK = wbase + stage * 2 * BLK;
@@ -317,7 +325,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       ldm_x4(smem_addr(sK + (lane & 15) * LDS + k * 16 + (lane >> 4) * 8), a0, a1, a2, a3);
       mma16816<T>(sc, a0, a1, a2, a3, qb[k][0], qb[k][1]);
     }
-    const int tok0 = (p_first + warp + 4 * i) * PAGE + g;
+    const int tok0 = (p_first + pw + WPH * i) * PAGE + g;
     const bool v0 = tok0 >= t_begin && tok0 < t_end, v1 = tok0 + 8 >= t_begin && tok0 + 8 < t_end;
     float corr[2];
 #pragma unroll
@@ -371,6 +379,49 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
     __syncwarp();
     if (i + 2 < my_pages) issue(i + 2, stage);
   }
+  // final (O, m, l) of head column j, dim d: the output when the row has one split (after folding in the
+  // shared-prefix partial), else the split's partial
+  auto emit = [&](int j, int d, float M, float Lsum, float O) {
+    const int hq = h * G + j;
+    if (nsplit == 1) {
+      if (sbase) {  // fold in the shared-prefix pass (partial slot 0, written by the preceding launch)
+        const float* p0 = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
+        const float m0 = p0[DH], Mn = fmaxf(M, m0);
+        const float w0 = (m0 == -INFINITY) ? 0.f : exp2f(m0 - Mn), w1 = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
+        O = O * w1 + p0[d] * w0;
+        Lsum = Lsum * w1 + p0[DH + 1] * w0;
+      }
+      out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
+    } else {
+      float* pp = part + (((size_t)s * Hq + hq) * max_splits + sbase + split) * (DH + 2);
+      pp[d] = O;
+      if (d == 0) pp[DH] = M, pp[DH + 1] = Lsum;
+    }
+  };
+  if constexpr (WPH == 1) {
+    // the warp's own stage buffers are idle now (every copy was waited for): stage (m, l, O^T) there
+    float* wm = reinterpret_cast<float*>(wbase);  // [8] maxima, [8] sums, [DH][8] O^T
+    float* wl = wm + 8;
+    float* wo = wl + 8;
+    if (g == 0) {
+#pragma unroll
+      for (int j = 0; j < 2; ++j) wm[2 * t4 + j] = m[j], wl[2 * t4 + j] = l[j];
+    }
+#pragma unroll
+    for (int mt = 0; mt < KS; ++mt) {
+      wo[(mt * 16 + g) * 8 + 2 * t4] = o[mt][0];
+      wo[(mt * 16 + g) * 8 + 2 * t4 + 1] = o[mt][1];
+      wo[(mt * 16 + g + 8) * 8 + 2 * t4] = o[mt][2];
+      wo[(mt * 16 + g + 8) * 8 + 2 * t4 + 1] = o[mt][3];
+    }
+    __syncwarp();
+    if (!hvalid) return;
+    for (int idx = lane; idx < G * DH; idx += 32) {
+      const int j = idx / DH, d = idx % DH;
+      emit(j, d, wm[j], wl[j], wo[d * 8 + j]);
+    }
+    return;
+  }
   // merge the 4 warps' partial softmax states
   __syncthreads();
   float* sm = reinterpret_cast<float*>(smem_raw);            // [4][8] maxima
@@ -401,21 +452,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
       Lsum += sl[w * 8 + j] * wt;
       O += so[((size_t)w * DH + d) * 8 + j] * wt;
     }
-    const int hq = h * G + j;
-    if (nsplit == 1) {
-      if (sbase) {  // fold in the shared-prefix pass (partial slot 0, written by the preceding launch)
-        const float* p0 = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
-        const float m0 = p0[DH], Mn = fmaxf(M, m0);
-        const float w0 = (m0 == -INFINITY) ? 0.f : exp2f(m0 - Mn), w1 = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
-        O = O * w1 + p0[d] * w0;
-        Lsum = Lsum * w1 + p0[DH + 1] * w0;
-      }
-      out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Lsum);
-    } else {
-      float* pp = part + (((size_t)s * Hq + hq) * max_splits + sbase + split) * (DH + 2);
-      pp[d] = O;
-      if (d == 0) pp[DH] = M, pp[DH + 1] = Lsum;
-    }
+    emit(j, d, M, Lsum, O);
   }
 }
 
@@ -817,7 +854,7 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
 template <typename T, int DH, int G>
 sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
                            const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
-                           int shared_pos, cudaStream_t st) {
+                           int shared_pos, int max_len, cudaStream_t st) {
   // with a shared prefix: slot 0 of the partials is the prefix pass, position splits follow
   const int sbase = shared_pos > 0 ? 1 : 0;
   const int t_min = shared_pos;
@@ -840,13 +877,23 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
                                        (size_t)(64 + 4 * DH * 8) * sizeof(float));
   static bool attr_set = false;
   if (!attr_set) {
-    SR_CUDA(cudaFuncSetAttribute(k_decode_attn_tc<T, DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    SR_CUDA(cudaFuncSetAttribute(k_decode_attn_tc<T, DH, G, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    SR_CUDA(cudaFuncSetAttribute(k_decode_attn_tc<T, DH, G, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
-  dim3 grid(Hkv, b, max_splits - sbase);
-  launch_k(k_decode_attn_tc<T, DH, G>, grid, 128, smem, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
-                                                       scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
+  // suffixes of at most 8 pages: one warp per (kv head, slot)
+  int span = max_len - t_min;
+  if (window > 0) span = std::min(span, window);
+  if (max_len > 0 && span <= 8 * PAGE && max_splits - sbase == 1) {
+    dim3 grid((Hkv + 3) / 4, b, 1);
+    launch_k(k_decode_attn_tc<T, DH, G, 1>, grid, 128, smem, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens,
+             Hkv, scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
+  } else {
+    dim3 grid(Hkv, b, max_splits - sbase);
+    launch_k(k_decode_attn_tc<T, DH, G, 4>, grid, 128, smem, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens,
+             Hkv, scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
+  }
   SR_LAUNCH();
   if (max_splits - sbase > 1) {  // some row has several position splits (a lone split merges the prefix itself)
     launch_k(k_decode_combine<T, DH>, dim3(Hkv * G, b), DH, 0, st, part, lens, Hkv * G, window, max_splits, t_min, sbase,
@@ -906,7 +953,8 @@ size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits) {
 
 sr_status launch_decode_attention(int et, const void* q, const void* pool_layer, const int* pt, int pt_stride,
                                   const int* ids, const int* lens, int b, int Hq, int Hkv, int dh, int window,
-                                  void* out, float* part, int max_splits, cudaStream_t st, int shared_pos) {
+                                  void* out, float* part, int max_splits, cudaStream_t st, int shared_pos,
+                                  int max_len) {
   if (b == 0) return SR_OK;
   const int G = Hq / Hkv;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "decode attention: n_heads %% n_kv_heads != 0");
@@ -918,7 +966,7 @@ sr_status launch_decode_attention(int et, const void* q, const void* pool_layer,
 #define SR_DECT(T, D, GG)                                                                                          \
   if (dh == D && G == GG)                                                                                            \
     return decode_attn_tc_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
-                                      shared_pos, st);
+                                      shared_pos, max_len, st);
   if (et == SR_DT_F16) {
     SR_DECT(f16, 128, 4) SR_DECT(f16, 128, 1) SR_DECT(f16, 128, 2) SR_DECT(f16, 128, 8)
     SR_DECT(f16, 64, 1) SR_DECT(f16, 64, 4) SR_DECT(f16, 32, 1)

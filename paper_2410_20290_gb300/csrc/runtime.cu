@@ -697,7 +697,7 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
     {
       Scope sc(pf, SR_KC_ATTN_DECODE, st, attn_flops, attn_bytes);
       SR_TRY(launch_decode_attention(m.et, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
-                                     d.window, w.att, w.part, splits, st, shared_pos));
+                                     d.window, w.att, w.part, splits, st, shared_pos, max_len));
     }
     SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, st, pf, SR_KC_GEMM_DECODE));
     {
@@ -1276,7 +1276,7 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
   if (splits > 1) SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&part),
                                           decode_attention_part_floats(b, n_heads, head_dim, splits) * sizeof(float), st));
   sr_status s = launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
-                                        head_dim, window, out, part, splits, st, shared_pos);
+                                        head_dim, window, out, part, splits, st, shared_pos, mx);
   if (part) cudaFreeAsync(part, st);
   return s;
 }

@@ -171,6 +171,9 @@ def _round16(x, dt=si.DT_F16):
     (si.DT_F16, 32, 8, 128, 40, [300, 301, 305], 256),
     (si.DT_F16, 32, 8, 128, 0, [17, 18, 600], 16),
     (si.DT_BF16, 32, 8, 128, 0, [300, 900], 272),
+    # suffixes of at most 8 pages run one warp per (kv head, slot); 2 kv heads leave two warps idle
+    (si.DT_F16, 16, 2, 128, 0, [289, 300, 310, 390], 288),
+    (si.DT_F16, 32, 8, 128, 0, [257, 258, 270, 300, 384] * 40, 256),
 ])
 def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens, shared):
     rng = np.random.default_rng(dh + len(lens))
