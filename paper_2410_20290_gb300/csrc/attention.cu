@@ -650,8 +650,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
 // the decode kernels' log2-scaled convention); the suffix kernel folds it into its result when a row's
 // suffix is one split, k_decode_combine merges it with the split partials otherwise.
 // No causal mask is needed (every prefix position precedes the query); a window masks per row.
-template <typename T, int DH, int G>
-__global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, const T* __restrict__ pool,
+template <typename T, int DH, int G, int NW>
+__global__ void __launch_bounds__(NW * 32, 2) k_prefix_attn(const T* __restrict__ q, const T* __restrict__ pool,
                                                      const int* __restrict__ pt, int pt_stride,
                                                      const int* __restrict__ slot_ids,
                                                      const int* __restrict__ lens, int n, int S, int Hkv,
@@ -659,11 +659,12 @@ __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, co
                                                      float* __restrict__ part) {
   pdl_entry();
   constexpr int HPC = G < 4 ? G : 4;       // query heads per CTA
-  constexpr int CPC = 4 / HPC;             // 16-candidate blocks per CTA
+  constexpr int CPC = NW / HPC;            // 16-candidate blocks per CTA (one warp per 16 rows)
+  constexpr int NT = NW * 32;
   constexpr int LD = DH + 8;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   T* sQ = reinterpret_cast<T*>(smem_raw);
-  T* sKV = sQ + BQ * LD;                   // [stage][K | V][64][LD]
+  T* sKV = sQ + 16 * NW * LD;              // [stage][K | V][64][LD]
   const int Hq = Hkv * G;
   const int h = blockIdx.y / (G / HPC), hg0 = (blockIdx.y % (G / HPC)) * HPC;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
@@ -686,7 +687,7 @@ __global__ void __launch_bounds__(128) k_prefix_attn(const T* __restrict__ q, co
     T* dK = sKV + (size_t)(kb & 1) * 2 * BKV * LD;
     T* dV = dK + BKV * LD;
     const int kbase = kb * BKV, kcount = min(BKV, S - kbase);
-    for (int c = tid; c < BKV * (DH / 8); c += 128) {
+    for (int c = tid; c < BKV * (DH / 8); c += NT) {
       const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
       const bool ok = row < kcount;
       const int key = kbase + row;
@@ -860,14 +861,15 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
   const int t_min = shared_pos;
   if (sbase) {
     if (!part) return set_err(SR_ERR_INVALID_ARG, "decode attention: partial buffer missing for the prefix pass");
-    constexpr int HPC = G < 4 ? G : 4, CPC = 4 / HPC;
-    const size_t psmem = (size_t)(BQ + 4 * BKV) * (DH + 8) * sizeof(T);
+    // eight warps (128 query rows) per CTA share each staged K/V block
+    constexpr int NW = 8, HPC = G < 4 ? G : 4, CPC = NW / HPC;
+    const size_t psmem = (size_t)(16 * NW + 4 * BKV) * (DH + 8) * sizeof(T);
     static bool pattr = false;
     if (!pattr) {
-      SR_CUDA(cudaFuncSetAttribute(k_prefix_attn<T, DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem));
+      SR_CUDA(cudaFuncSetAttribute(k_prefix_attn<T, DH, G, NW>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem));
       pattr = true;
     }
-    launch_k(k_prefix_attn<T, DH, G>, dim3((b + 16 * CPC - 1) / (16 * CPC), Hkv * (G / HPC)), 128, psmem, st, 
+    launch_k(k_prefix_attn<T, DH, G, NW>, dim3((b + 16 * CPC - 1) / (16 * CPC), Hkv * (G / HPC)), NW * 32, psmem, st, 
         (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, b, shared_pos, Hkv,
         1.4426950408889634f / sqrtf((float)DH), window, max_splits, part);
     SR_LAUNCH();
