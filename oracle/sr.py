@@ -45,6 +45,7 @@ import numpy as np
 
 import sr_inputs as si
 from .pool import PagePool, pool_pages, private_pages_full
+from .logprob import mean_logprob, token_logprob
 from .sampler import sample_token
 from .select import cut_index, float_keys, select_round
 from .transformer import Decoder, Transformer
@@ -97,7 +98,11 @@ class SpeculativeRejection:
     def __init__(self, gen: Transformer, rm: Transformer, prompt, N: int, alpha: float, sched_kind: int,
                  taus=(), max_new: int = 64, temperature: float = 1.0, eos_bias: float = 0.0, eos_id: int = 0,
                  seed: int = 0, n_pool_pages: int = 0,
-                 token_hook: Optional[Callable] = None, accept_hook: Optional[Callable] = None):
+                 token_hook: Optional[Callable] = None, accept_hook: Optional[Callable] = None,
+                 reward: str = "model"):
+        if reward not in ("model", "logprob"):
+            raise ValueError("reward must be 'model' or 'logprob'")
+        self.reward = reward
         self.gen, self.rm = gen, rm
         self.prompt = [int(t) for t in prompt]
         self.N, self.alpha = N, float(np.float32(alpha))
@@ -128,9 +133,12 @@ class SpeculativeRejection:
         if self.token_hook is not None:
             tok = int(self.token_hook(i, g, tok, logits))
         self.tokens[i].append(tok)
+        self.lp_sum[i] += token_logprob(logits, tok)
         self.gen_tokens += 1
 
     def _score(self, ids):
+        if self.reward == "logprob":  # Section 5.3: mean log-probability under the generator itself
+            return np.array([mean_logprob(self.lp_sum[i], len(self.tokens[i])) for i in ids], np.float32)
         r = score_sequences(self.rm, self.prompt, [self.tokens[i] for i in ids])
         self.rm_tokens += sum(len(self.tokens[i]) for i in ids)
         return r
@@ -175,11 +183,12 @@ class SpeculativeRejection:
         P, N = len(self.prompt), self.N
         self.status = [LIVE] * N
         self.tokens: List[List[int]] = [[] for _ in range(N)]
+        self.lp_sum = [0.0] * N
         self.final_reward = np.full(N, np.nan, np.float32)
         self.rounds: List[Round] = []
         self.snapshots: List[dict] = []
         self.gen_tokens = 0
-        self.rm_tokens = P
+        self.rm_tokens = P if self.reward == "model" else 0
         shared = [self.pool.pop() for _ in range(P // PAGE)]
         self.page_table = [list(shared) for _ in range(N)]
         dec = Decoder(self.gen, N, P + self.max_new)
@@ -256,22 +265,26 @@ def run_workload(w: si.Workload, gen_w: dict, rm_w: dict, prompt, seed: int = 0,
     return sr.run()
 
 
-def best_of_n(gen: Transformer, rm: Transformer, prompt, N, max_new, temperature, eos_bias, eos_id, seed):
-    """Plain Best-of-N (Section 3): N independent responses, each decoded on its own, argmax of s."""
+def best_of_n(gen: Transformer, rm: Transformer, prompt, N, max_new, temperature, eos_bias, eos_id, seed,
+              reward: str = "model"):
+    """Plain Best-of-N (Section 3): N independent responses, each decoded on its own, argmax of s
+    (s = the reward model, or with reward="logprob" the mean log-probability of Section 5.3)."""
     P = len(prompt)
-    seqs, rewards = [], []
+    seqs, rewards, lps = [], [], []
     for i in range(N):
         dec = Decoder(gen, 1, P + max_new)
         hn = dec.prefill(prompt, [0])
         logits = gen.logits(hn[-1])
-        y = []
+        y, lp = [], 0.0
         for g in range(max_new):
             if g > 0:
                 logits = gen.logits(dec.step([0], [y[-1]], P + g - 1)[0])
             y.append(sample_token(logits, seed, i, g, temperature, eos_bias, eos_id))
+            lp += token_logprob(logits, y[-1])
             if y[-1] == eos_id:
                 break
         seqs.append(y)
-    rewards = score_sequences(rm, prompt, seqs)
+        lps.append(mean_logprob(lp, len(y)))
+    rewards = score_sequences(rm, prompt, seqs) if reward == "model" else np.array(lps, np.float32)
     best = int(np.argmax(float_keys(rewards)))
     return best, seqs[best], float(rewards[best]), seqs, rewards
