@@ -113,9 +113,11 @@ class OracleSample:
     reward model), i.e. assuming cost linear in layers.  Models are built once; each run is timed."""
     L, N, MAX_NEW, P = 1, 2, 4, 64
 
-    def __init__(self, w: si.Workload):
+    def __init__(self, w: si.Workload, alpha=None, reward: str = "model"):
         from oracle.transformer import Transformer
         self.w = w
+        self.alpha = w.alpha if alpha is None else alpha
+        self.reward = reward
         self.g = w.gen.replace(n_layers=self.L)
         self.r = w.rm.replace(n_layers=self.L)
         self.gen = Transformer(self.g, si.random_weights(self.g, 100, 0))
@@ -125,7 +127,8 @@ class OracleSample:
             layer = m.qkv_dim * m.d_model + m.d_model * m.n_heads * m.head_dim + \
                 (3 if m.gated else 2) * m.ffn_dim * m.d_model
             return m.n_layers * layer + (m.vocab * m.d_model if m.has_lm_head else m.d_model)
-        self.scale = (per_tok(w.gen) + per_tok(w.rm)) / (per_tok(self.g) + per_tok(self.r))
+        with_rm = reward == "model"  # the self-likelihood reward runs no reward model
+        self.scale = (per_tok(w.gen) + with_rm * per_tok(w.rm)) / (per_tok(self.g) + with_rm * per_tok(self.r))
         try:
             import threadpoolctl
             self.cores = sum(p.get("num_threads", 0) for p in threadpoolctl.threadpool_info()
@@ -138,11 +141,12 @@ class OracleSample:
         w = self.w
         prompt = w.prompt(prompt_index)[:self.P]
         t0 = time.perf_counter()
-        res = SpeculativeRejection(self.gen, self.rm, prompt, self.N, w.alpha, si.SCHED_FIXED, (2,), self.MAX_NEW,
-                                   w.temperature, w.eos_bias, w.eos_id, 0).run()
+        res = SpeculativeRejection(self.gen, self.rm, prompt, self.N, self.alpha, si.SCHED_FIXED, (2,), self.MAX_NEW,
+                                   w.temperature, w.eos_bias, w.eos_id, 0, reward=self.reward).run()
         dt = time.perf_counter() - t0
         return {"value": res.gen_tokens / dt / self.scale, "unit": UNIT, "cores": self.cores, "kind": "oracle",
-                "sample": (f"oracle Algorithm 1 on {w.name} widths with {self.L}/{w.gen.n_layers} layers, "
+                "sample": (f"oracle Algorithm 1 ({self.reward} reward, alpha {self.alpha}) on {w.name} widths with "
+                           f"{self.L}/{w.gen.n_layers} layers, "
                            f"N={self.N}, P={len(prompt)}, {self.MAX_NEW} new tokens, one round at 2: "
                            f"{res.gen_tokens} tokens in {dt:.1f} s on the host, scaled by 1/{self.scale:.1f} "
                            f"(matmul parameters per token, full / sample)")}
@@ -152,7 +156,7 @@ def run_reference(args, w):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    smp = OracleSample(w)
+    smp = OracleSample(w, args.alpha, args.reward)
     steps = []
     for k in range(args.warmup + args.steps):
         s = smp.run(k % max(1, w.n_prompts))
@@ -180,6 +184,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama8b_n1024", choices=sorted(si.WORKLOADS))
     ap.add_argument("--alpha", type=float, default=None, help="override the rejection rate (0 = Best-of-N)")
+    ap.add_argument("--reward", default="model", choices=["model", "logprob"],
+                    help="reward model, or the generator's mean log-probability (Section 5.3)")
     ap.add_argument("--e2e-steps", type=int, default=1)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--prof-period", type=int, default=8,
@@ -211,6 +217,7 @@ def main():
     torch.cuda.empty_cache()
     stream = torch.cuda.Stream()
     sr.sr_set_stream(ctx, stream)
+    sr.sr_set_reward(ctx, sr.SR_REWARD_LOGPROB if args.reward == "logprob" else sr.SR_REWARD_MODEL)
     n_prompts = max(1, w.n_prompts)
     prompts = [torch.from_numpy(w.prompt(i)).cuda() for i in range(n_prompts)]
     out_tok = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
@@ -323,7 +330,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 1), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "model": "Llama-3-8B-shaped generator + reward model (random-init bf16)",
-                   "N": w.N, "alpha": alpha, "schedule": "memory-triggered" if w.sched_kind else f"tau={w.taus}",
+                   "N": w.N, "alpha": alpha, "reward": args.reward, "schedule": "memory-triggered" if w.sched_kind else f"tau={w.taus}",
                    "kv_pool_bytes": w.pool_bytes, "max_new": w.max_new, "temperature": w.temperature,
                    "eos_bias": w.eos_bias, "global_batch": w.N * world, "seq_len": f"P~U[{w.prompt_len_min},"
                    f"{w.prompt_len}] + {w.max_new}", "parallelism": f"replicas x{world}",
@@ -339,7 +346,7 @@ def main():
         "clocks": clocks, "e2e": e2e,
     }
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = OracleSample(w).run(0)
+        line["cpu_baseline"] = OracleSample(w, alpha, args.reward).run(0)
     print(json.dumps(line), flush=True)
 
 

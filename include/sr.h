@@ -160,6 +160,16 @@ void sr_destroy(sr_ctx* ctx);
 const char* sr_last_error(void);
 /* Use `stream` (a cudaStream_t) for all later work of this context; NULL restores the context's stream. */
 sr_status sr_set_stream(sr_ctx* ctx, void* stream);
+/* Reward used by the rejection rounds and the final choice (Eq. partial.reward.set, Eq. output.SBoN):
+ *   SR_REWARD_MODEL   the reward model s of sr_init (default);
+ *   SR_REWARD_LOGPROB the self-likelihood objective of Section 5.3, s(Y) = ln p(Y | X) / len(Y)
+ *                     under the generator itself (softmax of the raw logits: temperature 1, no EOS
+ *                     bias), a partial response scored over its tau tokens.  The sampler keeps
+ *                     ln p per candidate in the same pass over the logits; no reward-model work
+ *                     runs (sr_stats.rm_tokens = 0).
+ * The kind is read when a batch starts (sr_generate, sr_batch_begin); errors: SR_ERR_INVALID_ARG. */
+enum { SR_REWARD_MODEL = 0, SR_REWARD_LOGPROB = 1 };
+sr_status sr_set_reward(sr_ctx* ctx, int kind);
 /* Per-kernel-class CUDA-event timing: 0 off; k >= 1 times one launch in k of each class (1: every
    launch; each timed launch adds two event records to the stream) and counts all of them.  Results
    land in sr_stats.kern_*.  Errors: SR_ERR_INVALID_ARG (null context, k < 0). */
@@ -236,10 +246,13 @@ void sr_batch_end(sr_ctx* ctx, sr_batch* batch);
 /* Gumbel-max sampling (Eq. auto-regressive realised as in the Section 3
  * sampling step): token[r] = argmax_v (logits[r][v] + eos_bias [v == eos_id]) / T + g_v,
  * g_v = -ln(-ln u_v), u_v from Philox4x32-10 keyed (seed; v/4, orig_ids[r], steps[r], 0).
- * logits: fp32, row r at logits + r * ld (ld = 0 broadcasts one row).  b rows. */
+ * logits: fp32, row r at logits + r * ld (ld = 0 broadcasts one row).  b rows.
+ * logprob_sum (device, nullable, indexed by orig_ids[r]): += ln softmax(logits[r])[token[r]] in
+ * float64 (Section 5.3 self-likelihood; raw logits, NaN = -inf). */
 sr_status sr_k_sample(const float* logits, long long ld, int b, int vocab, const int32_t* orig_ids,
                       const int32_t* steps, uint64_t seed, float temperature, float eos_bias, int eos_id,
-                      int32_t* tokens_out, void* stream);
+                      int32_t* tokens_out, void* stream,
+                      double* logprob_sum);
 
 /* r_cut selection (Eqs. cutoff.threshold, accepted.set) on b <= 4096 fp32
  * rewards: k = min(floor(alpha b), b - 1) (or k_override >= 0); r_cut = k-th

@@ -90,7 +90,8 @@ _SIG = {
     "sr_reject_compact": [_P, _P, _P, _F, _P, _P, _P, _P],
     "sr_batch_query": [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P],
     "sr_batch_end": [_P, _P],
-    "sr_k_sample": [_P, ctypes.c_longlong, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P],
+    "sr_k_sample": [_P, ctypes.c_longlong, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P, _P],
+    "sr_set_reward": [_P, _I],
     "sr_k_rcut": [_P, _I, _F, _I, _P, _P, _P],
     "sr_k_gemm": [_I, _P, _P, _P, _I, _I, _I, _I, _P],
     "sr_k_decode_attention": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P],
@@ -177,6 +178,14 @@ def sr_destroy(ctx):
     LIB.sr_destroy(ctx)
 
 
+SR_REWARD_MODEL, SR_REWARD_LOGPROB = 0, 1
+
+
+def sr_set_reward(ctx, kind: int):
+    """SR_REWARD_MODEL (reward model) or SR_REWARD_LOGPROB (mean log-probability under the generator)."""
+    _check(LIB.sr_set_reward(ctx, int(kind)))
+
+
 def sr_set_profiling(ctx, period: int = 1):
     """0 / False: off; k >= 1: time one launch in k of each kernel class (True = every launch)."""
     _check(LIB.sr_set_profiling(ctx, int(period)))
@@ -259,9 +268,10 @@ def sr_batch_end(ctx, batch):
     LIB.sr_batch_end(ctx, batch)
 
 
-def sr_k_sample(logits, ld, b, vocab, orig_ids, steps, seed, temperature, eos_bias, eos_id, tokens_out, stream=None):
+def sr_k_sample(logits, ld, b, vocab, orig_ids, steps, seed, temperature, eos_bias, eos_id, tokens_out, stream=None,
+                logprob_sum=None):
     _check(LIB.sr_k_sample(_ptr(logits), ld, b, vocab, _ptr(orig_ids), _ptr(steps), seed, temperature, eos_bias,
-                           eos_id, _ptr(tokens_out), _stream(stream)))
+                           eos_id, _ptr(tokens_out), _stream(stream), _ptr(logprob_sum)))
 
 
 def sr_k_rcut(rewards, b, alpha, k_override, r_cut_out, mask_out, stream=None):

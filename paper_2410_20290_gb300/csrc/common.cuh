@@ -188,7 +188,8 @@ sr_status launch_copy_page(int dtype, void* pool, long long layer_stride_elems, 
 // sample.cu
 sr_status launch_sample(const float* logits, long long ld, int b, int V, const int* orig_ids, const int* steps,
                         uint64_t seed, float temperature, float eos_bias, int eos_id, int* tokens_out,
-                        int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st);
+                        int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st,
+                        double* lp_sum = nullptr);  // lp_sum: += ln p(token) per candidate id (Section 5.3 reward)
 
 // attention.cu
 // shared_pos > 0: positions [0, shared_pos) sit in pages shared by every row's page table (the prompt);

@@ -452,6 +452,10 @@ struct sr_ctx {
       *prompt_row = nullptr, *ids = nullptr, *prompt = nullptr, *iota = nullptr, *meta = nullptr, *out_tok = nullptr,
       *last_row = nullptr;
   float *reward = nullptr, *rr = nullptr, *logits = nullptr, *logits0 = nullptr;
+  // self-likelihood reward (Section 5.3): running ln p(Y | X) per candidate id
+  int reward_kind = SR_REWARD_MODEL;
+  double* lp_sum = nullptr;
+  size_t c_lpsum = 0;
   uint8_t* mask = nullptr;
   int* ctrl = nullptr;       // C_N ints
   float* ctrlf = nullptr;    // 4 floats (r_cut, score)
@@ -469,6 +473,7 @@ struct sr_batch {
   uint64_t seed = 0;
   int n_live = 0, n_rset = 0, g = 0;  // g: tokens generated by every live candidate
   bool active = false;
+  int reward_kind = SR_REWARD_MODEL;  // the context's reward kind when the batch started
 };
 
 namespace sr {
@@ -534,6 +539,7 @@ sr_status prepare_state(sr_ctx* c, sr_batch& b) {
   SR_TRY(grow(c->prompt_row, c->c_prow, (size_t)b.max_pages));
   SR_TRY(grow(c->ids, c->c_ids, N));
   SR_TRY(grow(c->reward, c->c_reward, N));
+  SR_TRY(grow(c->lp_sum, c->c_lpsum, N));
   SR_TRY(grow(c->rr, c->c_rr, N));
   SR_TRY(grow(c->mask, c->c_mask, N));
   SR_TRY(grow(c->last_row, c->c_lastrow, N));
@@ -550,6 +556,7 @@ sr_status prepare_state(sr_ctx* c, sr_batch& b) {
   }
   SR_CUDA(cudaMemsetAsync(c->status, 0xff, N * sizeof(int), c->st));
   SR_CUDA(cudaMemsetAsync(c->len, 0, N * sizeof(int), c->st));
+  SR_CUDA(cudaMemsetAsync(c->lp_sum, 0, N * sizeof(double), c->st));
   SR_CUDA(cudaMemsetAsync(c->pt, 0, N * b.max_pages * sizeof(int), c->st));
   return SR_OK;
 }
@@ -581,20 +588,22 @@ sr_status prefill_prompt(sr_ctx* c, sr_batch& b) {
   const Model& g = c->gen;
   const Model& r = c->rm;
   const int P = b.P;
-  // reward model
-  const size_t rm_layer = (size_t)P * r.kv_tok_elems() * r.esz;
-  SR_TRY(grow(c->rm_pk, c->c_rm_pk, rm_layer * r.d.n_layers));
-  SR_TRY(grow(c->rm_pv, c->c_rm_pv, rm_layer * r.d.n_layers));
   PrefillPlan plan;
   SR_TRY(upload_single_plan(c, P, plan));
-  PrefillKv kv;
-  kv.store_k = c->rm_pk;
-  kv.store_v = c->rm_pv;
-  kv.store_layer_bytes = rm_layer;
   Prof* pf = &c->prof;
   const std::vector<int> ptau(1, P);
-  SR_TRY(forward_prefill(r, c->wr, P, c->prompt, c->iota, plan, kv, c->st, pf, SR_KC_GEMM_PROMPT,
-                         prefill_attn_flops(r, ptau, 0, 1, 0)));
+  // reward model: prompt KV stored for the scoring passes (the self-likelihood reward needs none)
+  if (b.reward_kind == SR_REWARD_MODEL) {
+    const size_t rm_layer = (size_t)P * r.kv_tok_elems() * r.esz;
+    SR_TRY(grow(c->rm_pk, c->c_rm_pk, rm_layer * r.d.n_layers));
+    SR_TRY(grow(c->rm_pv, c->c_rm_pv, rm_layer * r.d.n_layers));
+    PrefillKv kv;
+    kv.store_k = c->rm_pk;
+    kv.store_v = c->rm_pv;
+    kv.store_layer_bytes = rm_layer;
+    SR_TRY(forward_prefill(r, c->wr, P, c->prompt, c->iota, plan, kv, c->st, pf, SR_KC_GEMM_PROMPT,
+                           prefill_attn_flops(r, ptau, 0, 1, 0)));
+  }
   // generator: pages for the prompt, KV into them
   {
     Scope sc(pf, SR_KC_CONTROL, c->st);
@@ -635,7 +644,8 @@ sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
   {
     Scope sc(pf, SR_KC_SAMPLE, c->st, 0, 4.0 * g.d.vocab);
     SR_TRY(launch_sample(c->logits0, 0, count, g.d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias,
-                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, c->st));
+                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, c->st,
+                         b.reward_kind == SR_REWARD_LOGPROB ? c->lp_sum : nullptr));
   }
   {
     Scope sc(pf, SR_KC_CONTROL, c->st);
@@ -717,7 +727,8 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
   {
     Scope sc(pf, SR_KC_SAMPLE, st, 0, 4.0 * n * d.vocab);
     SR_TRY(launch_sample(c->logits, d.vocab, n, d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias,
-                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, st));
+                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, st,
+                         b.reward_kind == SR_REWARD_LOGPROB ? c->lp_sum : nullptr));
   }
   {
     Scope sc(pf, SR_KC_CONTROL, st);
@@ -741,6 +752,15 @@ __global__ void k_gather_rows(const int* __restrict__ ids, const int* __restrict
   if (threadIdx.x == 0) last_row[j] = r0 + n - 1;
 }
 
+// Self-likelihood reward of Section 5.3: s = ln p(Y^{<=tau} | X) / tau from the running sums the sampler
+// keeps per candidate (tau = the tokens the candidate has, as for the reward model).
+__global__ void k_mean_logprob(const int* __restrict__ ids_taus, int n, const double* __restrict__ lp_sum,
+                               float* __restrict__ out) {
+  pdl_entry();
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j < n) out[j] = (float)(lp_sum[ids_taus[j]] / (double)ids_taus[n + j]);
+}
+
 constexpr int CHUNK_ROWS = 16384;  // reward-model rows (response tokens) per scoring pass
 
 // Rewards s(X ++ Y_k^{<= tau_k}) for candidates ids_h[0..n) with tau_k = taus[k] (Eq.
@@ -751,6 +771,18 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
   const Model& r = c->rm;
   const int n = (int)ids_h.size();
   if (n == 0) return SR_OK;
+  if (b.reward_kind == SR_REWARD_LOGPROB) {
+    SR_CUDA(cudaStreamSynchronize(c->st));  // the pinned staging buffer may still feed an earlier copy
+    SR_TRY(grow_host(c->h_meta, c->c_hmeta, 2 * (size_t)n));
+    SR_TRY(grow(c->meta, c->c_meta, 2 * (size_t)n));
+    for (int j = 0; j < n; ++j) c->h_meta[j] = ids_h[j], c->h_meta[n + j] = taus[j];
+    SR_CUDA(cudaMemcpyAsync(c->meta, c->h_meta, 2 * (size_t)n * sizeof(int), cudaMemcpyHostToDevice, c->st));
+    Scope sc(&c->prof, SR_KC_CONTROL, c->st);
+    launch_k(k_mean_logprob, (n + 255) / 256, 256, 0, c->st, (const int*)c->meta, n, (const double*)c->lp_sum,
+             rewards_dev);
+    SR_LAUNCH();
+    return SR_OK;
+  }
   const size_t rm_layer = (size_t)b.P * r.kv_tok_elems() * r.esz;
   // plan chunks on the host: [ids | off | tiles_seq | tiles_q0] per chunk in one pinned buffer
   struct Chunk {
@@ -865,6 +897,7 @@ sr_status begin(sr_ctx* c, sr_batch& b, const int32_t* prompt, bool prompt_on_de
   SR_TRY(validate_common(c, P, N, max_new, temperature, eos_id));
   c->prof.reset();
   b = sr_batch();
+  b.reward_kind = c->reward_kind;
   b.P = P, b.N = N, b.max_new = max_new, b.temperature = temperature, b.eos_bias = eos_bias, b.eos_id = eos_id;
   b.seed = seed;
   b.n_sh = P / PAGE;
@@ -970,6 +1003,7 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
     S.ms_score += now_ms() - tf;
   }
   S.rm_tokens += b.P;
+  if (b.reward_kind != SR_REWARD_MODEL) S.rm_tokens = 0;  // the generator scored itself
   SR_TRY(ctl_final(b.N, c->status, c->reward, c->tok, b.max_new, c->len, c->out_tok, c->d_outlen, c->ctrlf + 1,
                    c->ctrl, c->st));
   SR_TRY(read_ctrl(c));
@@ -1068,6 +1102,13 @@ void sr_destroy(sr_ctx* c) {
   if (c->h_meta) cudaFreeHost(c->h_meta);
   if (c->own) cudaStreamDestroy(c->own);
   delete c;
+}
+
+sr_status sr_set_reward(sr_ctx* c, int kind) {
+  if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
+  if (kind != SR_REWARD_MODEL && kind != SR_REWARD_LOGPROB) return set_err(SR_ERR_INVALID_ARG, "unknown reward kind");
+  c->reward_kind = kind;
+  return SR_OK;
 }
 
 sr_status sr_set_profiling(sr_ctx* c, int enable) {
@@ -1233,11 +1274,11 @@ void sr_batch_end(sr_ctx* c, sr_batch* b) {
 // ---- kernel-level entry points ----
 sr_status sr_k_sample(const float* logits, long long ld, int b, int vocab, const int32_t* orig_ids,
                       const int32_t* steps, uint64_t seed, float temperature, float eos_bias, int eos_id,
-                      int32_t* tokens_out, void* stream) {
+                      int32_t* tokens_out, void* stream, double* logprob_sum) {
   if (!logits || !orig_ids || !steps || !tokens_out || b < 0 || vocab < 1)
     return set_err(SR_ERR_INVALID_ARG, "sr_k_sample: bad argument");
   return launch_sample(logits, ld, b, vocab, orig_ids, steps, seed, temperature, eos_bias, eos_id, tokens_out,
-                       nullptr, 0, nullptr, nullptr, static_cast<cudaStream_t>(stream));
+                       nullptr, 0, nullptr, nullptr, static_cast<cudaStream_t>(stream), logprob_sum);
 }
 
 sr_status sr_k_rcut(const float* rewards, int b, float alpha, int k_override, float* r_cut_out, uint8_t* mask_out,

@@ -12,6 +12,10 @@
 //
 // One block per row; each thread handles groups of 4 consecutive vocabulary ids (one Philox
 // call per group); block argmax with ties to the lowest id; NaN logits count as -inf.
+//
+// With `lp_sum` set, the same pass also takes ln sum_v exp(logit_v) of the raw logits (online
+// max / rescaled sum) and adds ln p(token) = logit_token - that to lp_sum[candidate id]: the running
+// ln p(Y | X) of the self-likelihood reward of Section 5.3 (temperature 1, no EOS bias).
 #include "common.cuh"
 
 namespace sr {
@@ -67,10 +71,12 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
                                                     const int* __restrict__ orig_ids, const int* __restrict__ steps,
                                                     uint32_t k0, uint32_t k1, float temperature, float eos_bias,
                                                     int eos_id, int* __restrict__ tokens_out, int* tok_hist,
-                                                    int max_new, int* lens, int* status) {
+                                                    int max_new, int* lens, int* status, double* lp_sum) {
   pdl_entry();
   __shared__ float s_best[THREADS / 32];
   __shared__ int s_idx[THREADS / 32];
+  __shared__ float s_m[THREADS / 32], s_s[THREADS / 32];
+  float lm = -__int_as_float(0x7f800000), ls = 0.f;  // running max and sum exp(l - max) of the raw logits
   const int r = blockIdx.x;
   const int id = orig_ids[r];
   const int step = steps ? steps[r] : lens[id];
@@ -97,6 +103,14 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
       const int v = v0 + j;
       if (v >= V) break;
       float a = l[j];
+      if (lp_sum && a == a) {
+        if (a > lm) {
+          ls = ls * expf(lm - a) + 1.f;
+          lm = a;
+        } else {
+          ls += expf(a - lm);
+        }
+      }
       if (v == eos_id) a = __fadd_rn(a, eos_bias);
       if (a != a) a = -__int_as_float(0x7f800000);
       const float z = __fadd_rn(__fmul_rn(a, inv_t), gumbel_of(words[j]));
@@ -111,11 +125,33 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
     if (ob > best || (ob == best && ov < best_v)) best = ob, best_v = ov;
   }
   if ((threadIdx.x & 31) == 0) s_best[threadIdx.x >> 5] = best, s_idx[threadIdx.x >> 5] = best_v;
+  if (lp_sum) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float om = __shfl_xor_sync(0xffffffffu, lm, o), os = __shfl_xor_sync(0xffffffffu, ls, o);
+      const float mn = fmaxf(lm, om);
+      ls = (mn == -__int_as_float(0x7f800000)) ? 0.f : ls * expf(lm - mn) + os * expf(om - mn);
+      lm = mn;
+    }
+    if ((threadIdx.x & 31) == 0) s_m[threadIdx.x >> 5] = lm, s_s[threadIdx.x >> 5] = ls;
+  }
   __syncthreads();
   if (threadIdx.x == 0) {
     for (int w = 1; w < THREADS / 32; ++w)
       if (s_best[w] > best || (s_best[w] == best && s_idx[w] < best_v)) best = s_best[w], best_v = s_idx[w];
     if (best_v == 0x7fffffff) best_v = 0;  // every perturbed logit was -inf / NaN: id 0
+    if (lp_sum) {
+      float M = s_m[0], S = s_s[0];
+      for (int w = 1; w < THREADS / 32; ++w) {
+        const float mn = fmaxf(M, s_m[w]);
+        S = (mn == -__int_as_float(0x7f800000)) ? 0.f : S * expf(M - mn) + s_s[w] * expf(s_m[w] - mn);
+        M = mn;
+      }
+      const float lt = row[best_v];
+      const double lp = (lt != lt || M == -__int_as_float(0x7f800000)) ? -INFINITY
+                                                                         : (double)lt - ((double)M + log((double)S));
+      lp_sum[id] += lp;
+    }
     if (tokens_out) tokens_out[r] = best_v;
     if (tok_hist) {
       tok_hist[(size_t)id * max_new + step] = best_v;
@@ -129,12 +165,12 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
 
 sr_status launch_sample(const float* logits, long long ld, int b, int V, const int* orig_ids, const int* steps,
                         uint64_t seed, float temperature, float eos_bias, int eos_id, int* tokens_out, int* tok_hist,
-                        int max_new, int* lens, int* status, cudaStream_t st) {
+                        int max_new, int* lens, int* status, cudaStream_t st, double* lp_sum) {
   if (b == 0) return SR_OK;
   if (!(temperature > 0.f)) return set_err(SR_ERR_INVALID_ARG, "temperature must be > 0");
   launch_k(k_sample, b, THREADS, 0, st, logits, ld, V, orig_ids, steps, (uint32_t)(seed & 0xFFFFFFFFu),
                                   (uint32_t)(seed >> 32), temperature, eos_bias, eos_id, tokens_out, tok_hist, max_new,
-                                  lens, status);
+                                  lens, status, lp_sum);
   SR_LAUNCH();
   return SR_OK;
 }
