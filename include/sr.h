@@ -160,6 +160,15 @@ void sr_destroy(sr_ctx* ctx);
 const char* sr_last_error(void);
 /* Use `stream` (a cudaStream_t) for all later work of this context; NULL restores the context's stream. */
 sr_status sr_set_stream(sr_ctx* ctx, void* stream);
+/* b_init of Algorithm 1's first step ("based on the GPU memory capacity and the prompt length"): the
+ * largest N <= n_max whose candidates can all generate tau_min tokens in a pool of kv_pool_bytes (pages
+ * as in sr_init: floor(bytes / (16 positions x KV bytes per position of `gen`))) before the first
+ * memory-triggered round -- pages - floor(P / 16) shared prompt pages, divided by the private pages one
+ * candidate holds after tau_min tokens.  Host-only arithmetic.  *n_out gets the value (0 when nothing fits).
+ * Errors: SR_ERR_INVALID_ARG (null or non-positive argument), SR_ERR_OOM (*n_out = 0). */
+sr_status sr_auto_b_init(const sr_model_desc* gen, size_t kv_pool_bytes, int P, int tau_min, int n_max,
+                         int* n_out);
+
 /* Reward used by the rejection rounds and the final choice (Eq. partial.reward.set, Eq. output.SBoN):
  *   SR_REWARD_MODEL   the reward model s of sr_init (default);
  *   SR_REWARD_LOGPROB the self-likelihood objective of Section 5.3, s(Y) = ln p(Y | X) / len(Y)

@@ -51,3 +51,17 @@ def private_pages_full(P: int, max_new: int, page_tokens: int = 16) -> int:
     never fed back)."""
     last = P + max_new - 2
     return last // page_tokens + 1 - P // page_tokens
+
+
+def auto_b_init(n_pages: int, P: int, tau_min: int, n_max: int, page_tokens: int = 16) -> int:
+    """Initial batch size of Algorithm 1's first step ("based on the GPU memory capacity and the prompt
+    length"), read as: the largest N <= n_max whose candidates can all generate tau_min tokens before the pool
+    runs out, i.e. before the first memory-triggered round.  The prompt's full pages are shared; each candidate
+    then holds private_pages_full(P, tau_min) pages.  0 when not even one candidate fits."""
+    avail = n_pages - P // page_tokens
+    per = private_pages_full(P, tau_min, page_tokens)
+    if avail < 0:
+        return 0
+    if per == 0:
+        return n_max
+    return min(n_max, avail // per)

@@ -92,6 +92,7 @@ _SIG = {
     "sr_batch_end": [_P, _P],
     "sr_k_sample": [_P, ctypes.c_longlong, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P, _P],
     "sr_set_reward": [_P, _I],
+    "sr_auto_b_init": [_P, ctypes.c_size_t, _I, _I, _I, _P],
     "sr_k_rcut": [_P, _I, _F, _I, _P, _P, _P],
     "sr_k_gemm": [_I, _P, _P, _P, _I, _I, _I, _I, _P],
     "sr_k_decode_attention": [_I, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P],
@@ -179,6 +180,17 @@ def sr_destroy(ctx):
 
 
 SR_REWARD_MODEL, SR_REWARD_LOGPROB = 0, 1
+
+
+def sr_auto_b_init(gen, kv_pool_bytes: int, P: int, tau_min: int, n_max: int) -> int:
+    """Largest N <= n_max that reaches tau_min tokens before the first memory-triggered round."""
+    d = make_desc(gen)
+    n = ctypes.c_int(0)
+    st = LIB.sr_auto_b_init(ctypes.byref(d), kv_pool_bytes, P, tau_min, n_max, ctypes.byref(n))
+    if st == SR_ERR_OOM:
+        return 0
+    _check(st)
+    return n.value
 
 
 def sr_set_reward(ctx, kind: int):

@@ -1104,6 +1104,22 @@ void sr_destroy(sr_ctx* c) {
   delete c;
 }
 
+sr_status sr_auto_b_init(const sr_model_desc* gen, size_t kv_pool_bytes, int P, int tau_min, int n_max,
+                         int* n_out) {
+  if (!gen || !n_out) return set_err(SR_ERR_INVALID_ARG, "null argument");
+  if (P < 1 || tau_min < 1 || n_max < 1 || gen->n_layers < 1 || gen->n_kv_heads < 1 || gen->head_dim < 1)
+    return set_err(SR_ERR_INVALID_ARG, "sr_auto_b_init: bad argument");
+  const size_t esz = gen->dtype == SR_DT_F32 ? 4 : 2;
+  const size_t kvt = (size_t)gen->n_layers * 2 * gen->n_kv_heads * gen->head_dim * esz;
+  const long long pages = (long long)(kv_pool_bytes / (PAGE * kvt));
+  const long long avail = pages - P / PAGE;
+  const int per = private_pages_full(P, tau_min);
+  long long n = avail < 0 ? 0 : (per == 0 ? n_max : std::min<long long>(n_max, avail / per));
+  *n_out = (int)n;
+  if (n < 1) return set_err(SR_ERR_OOM, "sr_auto_b_init: the pool cannot hold one candidate to tau_min tokens");
+  return SR_OK;
+}
+
 sr_status sr_set_reward(sr_ctx* c, int kind) {
   if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
   if (kind != SR_REWARD_MODEL && kind != SR_REWARD_LOGPROB) return set_err(SR_ERR_INVALID_ARG, "unknown reward kind");
