@@ -12,15 +12,17 @@
 //                 (~192 KB of shared memory in flight per SM)
 //   warp 1      : allocates 2*BN TMEM columns; one elected lane issues tcgen05.mma (M=128, N=BN,
 //                 K=16) and tcgen05.commit to release smem stages / publish accumulators
-//   warps 2..5  : epilogue -- tcgen05.ld 32 lanes x 32 columns per warp (the warp's TMEM lane
-//                 quadrant is warp % 4), fused conversion / residual add / gated activation,
+//   warps 2..5  : epilogue -- tcgen05.ld 32 lanes x 64 columns per warp and wait (the warp's TMEM
+//                 lane quadrant is warp % 4), fused conversion / residual add / gated activation,
 //                 direct global stores
 // Two BN-column accumulators let the epilogue of tile i overlap the mainloop of tile i+1.
 // Tiles are walked M-fastest so that the CTAs running at the same time share W tiles in L2.
 // Two variants raise the MMA work per staged byte (the limit of the 128-row tiles on GB300):
 // 256 x 256 tiles on one SM (two M = 128 MMAs per W tile, single-buffered accumulator), and
 // 256 x 256 tiles on a CTA pair (cta_group::2, M = 256 MMAs, each SM staging half of A and W,
-// double-buffered accumulators).  The launcher picks among the three per shape.
+// double-buffered accumulators).  Decode batches of at most 512 rows can instead run the product
+// transposed (C^T = W A^T) on a CTA pair, every activation row on the MMA's N side, with the K range
+// split over the SMs and the fp32 partials summed in slice order.  The launcher picks per shape.
 // Every mbarrier wait is bounded (about 2 s of %globaltimer); on expiry the CTA records an error,
 // drains its own TMA copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
