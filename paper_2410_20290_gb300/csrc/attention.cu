@@ -644,7 +644,7 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
 
 // Shared-prompt prefix of decode attention.  Positions [0, S) sit in pages every live candidate shares
 // (the prompt's full pages), so instead of each candidate re-reading them, one CTA takes the queries of
-// several candidates for up to 4 query heads of one kv head (64 query rows, one warp per 16 rows) and runs
+// several candidates for up to 4 query heads of one kv head (NW warps of 16 query rows each) and runs
 // flash attention over the prefix keys with mma.sync; each 64-position K/V block is loaded once per CTA
 // through a 2-stage cp.async pipeline.  The result is written unnormalised as partial slot 0 (O, m, l in
 // the decode kernels' log2-scaled convention); the suffix kernel folds it into its result when a row's
