@@ -51,3 +51,23 @@ def test_errors_without_device(lib_path):
     with pytest.raises(b.SrError) as e:
         b.sr_init(m.replace(n_heads=3, n_kv_heads=2), x, m.replace(has_lm_head=0, has_scalar_head=1), x)
     assert e.value.status in (b.SR_ERR_UNSUPPORTED, b.SR_ERR_INVALID_ARG)
+
+
+def test_host_only_entry_points_validate_arguments(lib_path):
+    """Calls that do no device work check their arguments on the host: null contexts and impossible sizes."""
+    from paper_2410_20290_gb300 import binding as b
+    import sr_inputs as si
+    m = si.WORKLOADS["llama8b_n1024"].gen
+    for kind in (b.SR_REWARD_MODEL, b.SR_REWARD_LOGPROB):
+        with pytest.raises(b.SrError) as e:
+            b.sr_set_reward(None, kind)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+    with pytest.raises(b.SrError) as e:
+        b.sr_set_profiling(None, 8)
+    assert e.value.status == b.SR_ERR_INVALID_ARG
+    for P, tau, n_max in ((0, 8, 16), (16, 0, 16), (16, 8, 0)):
+        with pytest.raises(b.SrError) as e:
+            b.sr_auto_b_init(m, 60 * 10 ** 9, P, tau, n_max)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+    assert b.sr_auto_b_init(m, 1000, 16, 8, 16) == 0          # a pool below one page: nothing fits (SR_ERR_OOM)
+    assert "tau_min" in b.LIB.sr_last_error().decode()
