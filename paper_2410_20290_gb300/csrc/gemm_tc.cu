@@ -1021,7 +1021,9 @@ int g_tm_override = 0;  // SR_GEMM_TM: force the tile height (128 or 256)
 int g_pair_override = -1;  // SR_GEMM_PAIR: 1 forces the CTA-pair kernel, 0 forbids it
 int g_skinny_override = -1;  // SR_GEMM_SKINNY: 0 forbids the skinny kernel (else used for M <= 512)
 std::mutex g_ws_mu;
-std::map<int, std::pair<float*, size_t>> g_ws;  // per device: split-K partial workspace (floats)
+// split-K partial workspace (floats) per (device, stream): launches on one stream run in order, so one
+// buffer per stream keeps contexts on different streams from sharing it
+std::map<std::pair<int, cudaStream_t>, std::pair<float*, size_t>> g_ws;
 int* g_err = nullptr;
 
 // Estimated relative time of a tile width: waves of persistent CTAs x per-tile cost.  The per-tile
@@ -1133,11 +1135,11 @@ sr_status launch_pair(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArg
 
 sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, int K, int box_rows);
 
-sr_status skinny_workspace(size_t floats, float** out) {
+sr_status skinny_workspace(size_t floats, cudaStream_t st, float** out) {
   int dev;
   SR_CUDA(cudaGetDevice(&dev));
   std::lock_guard<std::mutex> lk(g_ws_mu);
-  auto& w = g_ws[dev];
+  auto& w = g_ws[std::make_pair(dev, st)];
   if (w.second < floats) {
     if (w.first) SR_CUDA(cudaFree(w.first));
     w.first = nullptr;
@@ -1212,7 +1214,7 @@ sr_status launch_skinny(const void* A, const void* W, bool bf, const EpiArgs& ep
   SR_TRY(encode_kmajor(&tw, W, bf, N, K, BM));
   SR_TRY(encode_kmajor(&ta, A, bf, M, K, g.Np / 2));
   float* part = nullptr;
-  if (g.s_split > 1) SR_TRY(skinny_workspace((size_t)g.s_split * M * N, &part));
+  if (g.s_split > 1) SR_TRY(skinny_workspace((size_t)g.s_split * M * N, st, &part));
   const int units = g.n_tiles * g.s_split;
   const int pairs = std::min(units, max_pairs);
   const size_t smem = 1024 + (size_t)g.stages * g.stage_bytes + PairCfg<256>::GUARD + BAR_BYTES;
