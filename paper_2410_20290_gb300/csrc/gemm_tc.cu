@@ -134,22 +134,6 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
-// commit that arrives on the barrier at this smem offset in every CTA of `mask` in the cluster
-__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-                   smem_u32(bar)),
-               "h"(mask)
-               : "memory");
-}
-// 2D TMA load written to the same smem offset in every CTA of `mask`, signalling each CTA's barrier
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
-                                               uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, "
-      "{%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
-      : "memory");
-}
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -341,12 +325,7 @@ __device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int
   }
 }
 
-// CL = 2: the kernel runs in clusters of two CTAs that take the two M tiles of a pair with the same W
-// tile; each CTA loads half of the W tile and multicasts it to both, so the L2 -> SM traffic per stage
-// drops from 48 KB to 32 KB (BN = 256).  Stage release is signalled to both CTAs (empty barriers count
-// two commits).  When the M-tile count is odd, the last pair's second tile is all zero-filled rows that
-// the epilogue skips.
-template <int TM, int BN, int CL>
+template <int TM, int BN>
 __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
               int N, int K, int* err) {
@@ -354,7 +333,6 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   constexpr int A_BYTES = C::A_BYTES, B_BYTES = C::B_BYTES, STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES;
   constexpr int TMEM_COLS = C::TMEM_COLS, MH = C::MH, NACC = C::NACC, EPI_WARPS = C::EPI_WARPS;
   constexpr int ACC_COLS = MH * BN;  // TMEM columns of one accumulator buffer
-  static_assert(CL == 1 || CL == 2, "cluster size");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -371,16 +349,14 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   const uint32_t idesc = idesc_for(ep.bf != 0, BN);
   const int num_m = (M + TM - 1) / TM, num_n = (N + BN - 1) / BN;
   const int num_k = (K + BK - 1) / BK;
-  // tiles of this CTA: index t over (M-tile group of CL, N tile), M fastest; m tile = CL * group + rank
-  const int rank = CL == 2 ? (int)cluster_rank() : 0;
-  const int num_mg = (num_m + CL - 1) / CL, num_tiles = num_mg * num_n;
-  const int t0 = blockIdx.x / CL, tstep = gridDim.x / CL;
-  constexpr uint16_t MASK = CL == 2 ? 0x3 : 0x1;
+  // tiles of this CTA: index t over (M tile, N tile), M fastest
+  const int num_tiles = num_m * num_n;
+  const int t0 = blockIdx.x, tstep = gridDim.x;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], CL);
+      mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
@@ -399,7 +375,6 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (CL == 2) cluster_sync();  // the peer's barriers are initialised before anyone signals them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   pdl_entry();  // prologue done; the operands written by the previous kernel are visible from here
@@ -414,7 +389,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       for (int s = 0; s < STAGES; ++s) armed[s] = 0, armed_par[s] = 0;
       bool ok = true;
       for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
-        const int mb = (tile % num_mg) * CL + rank, nb = tile / num_mg;
+        const int mb = tile % num_m, nb = tile / num_m;
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
             ok = false;
@@ -422,11 +397,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
           }
           mbar_expect_tx(&full[stage], STAGE_BYTES);
           tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * TM);
-          if (CL == 2)
-            tma_load_2d_mc(sB + stage * B_BYTES + rank * (B_BYTES / 2), &tmB, &full[stage], kb * BK,
-                           nb * BN + rank * (BN / 2), MASK);
-          else
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * BN);
+          tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * BN);
           armed[stage] = 1;
           armed_par[stage] = phase;
           if (++stage == STAGES) stage = 0, phase ^= 1u;
@@ -470,8 +441,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
               umma(d_tmem + (uint32_t)(h * BN), a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc,
                    (kb | kk) != 0);
           }
-          if (CL == 2) umma_commit_mc(&empty[stage], MASK);
-          else umma_commit(&empty[stage]);
+          umma_commit(&empty[stage]);
           if (++stage == STAGES) stage = 0, phase ^= 1u;
         }
         if (!ok) break;
@@ -493,7 +463,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = t0; tile < num_tiles; tile += tstep) {
-      const int mb = (tile % num_mg) * CL + rank, nb = tile / num_mg;
+      const int mb = tile % num_m, nb = tile / num_m;
       // one lane waits and broadcasts, so the warp-collective tcgen05.ld below stays converged
       int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag) : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -516,7 +486,6 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (CL == 2) cluster_sync();  // no peer still writes into this CTA's shared memory or barriers
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
@@ -1016,13 +985,14 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 int g_num_sms = 0;
 int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
-int g_cl_override = 0;  // SR_GEMM_CL: force the cluster size (1 or 2)
 int g_tm_override = 0;  // SR_GEMM_TM: force the tile height (128 or 256)
 int g_pair_override = -1;  // SR_GEMM_PAIR: 1 forces the CTA-pair kernel, 0 forbids it
 int g_skinny_override = -1;  // SR_GEMM_SKINNY: 0 forbids the skinny kernel (else used for M <= 512)
 std::mutex g_ws_mu;
 // split-K partial workspace (floats) per (device, stream): launches on one stream run in order, so one
-// buffer per stream keeps contexts on different streams from sharing it
+// buffer per stream keeps contexts on different streams from sharing it.  sr_destroy frees the buffers
+// of the context's own and sr_set_stream streams; a stream passed only to sr_k_gemm or sr_generate_dev keeps
+// its buffer until process exit.
 std::map<std::pair<int, cudaStream_t>, std::pair<float*, size_t>> g_ws;
 int* g_err = nullptr;
 
@@ -1057,47 +1027,18 @@ bool pick_tall(int M, int N, int K) {
   return t_tall < t_small;
 }
 
-template <int TM, int BN, int CL>
+template <int TM, int BN>
 sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
                     cudaStream_t st) {
   using C = Cfg<TM, BN>;
-  static int max_groups = 0;
-  if (!max_groups) {
-    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM_BYTES));
-    max_groups = g_num_sms / CL;
-    if (CL > 1) {
-      SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN, CL>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0));
-      cudaLaunchConfig_t qc = {};
-      cudaLaunchAttribute qa[1];
-      qa[0].id = cudaLaunchAttributeClusterDimension;
-      qa[0].val.clusterDim.x = CL, qa[0].val.clusterDim.y = 1, qa[0].val.clusterDim.z = 1;
-      qc.gridDim = dim3(g_num_sms / CL * CL);
-      qc.blockDim = dim3(C::THREADS);
-      qc.dynamicSmemBytes = C::SMEM_BYTES;
-      qc.attrs = qa;
-      qc.numAttrs = 1;
-      int clusters = 0;
-      if (cudaOccupancyMaxActiveClusters(&clusters, k_gemm_tc<TM, BN, CL>, &qc) == cudaSuccess && clusters > 0)
-        max_groups = std::min(max_groups, clusters);
-      cudaGetLastError();
-    }
+  static int max_ctas = 0;
+  if (!max_ctas) {
+    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
+    max_ctas = g_num_sms;
   }
-  const int groups_total = ((M + TM * CL - 1) / (TM * CL)) * ((N + BN - 1) / BN);
-  const int groups = std::min(groups_total, max_groups);
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = CL, attr[0].val.clusterDim.y = 1, attr[0].val.clusterDim.z = 1;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
-  cfg.gridDim = dim3(groups * CL);
-  cfg.blockDim = dim3(C::THREADS);
-  cfg.dynamicSmemBytes = C::SMEM_BYTES;
-  cfg.stream = st;
-  cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  SR_CUDA(cudaLaunchKernelEx(&cfg, k_gemm_tc<TM, BN, CL>, ta, tb, ep, M, N, K, g_err));
+  const int tiles = ((M + TM - 1) / TM) * ((N + BN - 1) / BN);
+  launch_k(k_gemm_tc<TM, BN>, std::min(tiles, max_ctas), C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err);
+  SR_CUDA(cudaGetLastError());
   return SR_OK;
 }
 
@@ -1272,7 +1213,6 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     SR_CUDA(cudaMalloc(&g_err, sizeof(int)));
     SR_CUDA(cudaMemset(g_err, 0, sizeof(int)));
     if (const char* e = getenv("SR_GEMM_BN")) g_bn_override = atoi(e);
-    if (const char* e = getenv("SR_GEMM_CL")) g_cl_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_TM")) g_tm_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_PAIR")) g_pair_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_SKINNY")) g_skinny_override = atoi(e);
@@ -1280,11 +1220,11 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
   CUtensorMap ta, tb;
   EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
-  const bool forced = g_pair_override == 1 || g_bn_override != 0 || g_tm_override != 0 || g_cl_override != 0;
+  const bool forced = g_pair_override == 1 || g_bn_override != 0 || g_tm_override != 0;
   if (M <= 512 && g_skinny_override != 0 && (g_skinny_override == 1 || (!forced && pick_skinny(M, N, K))))
     return launch_skinny(A, W, bf, ep, M, N, K, st);
-  if (g_pair_override == 1 || (g_pair_override == -1 && g_bn_override == 0 && g_tm_override == 0 &&
-                               g_cl_override == 0 && pick_pair(M, N, K, gated))) {
+  if (g_pair_override == 1 ||
+      (g_pair_override == -1 && g_bn_override == 0 && g_tm_override == 0 && pick_pair(M, N, K, gated))) {
     SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
     SR_TRY(encode_kmajor(&tb, W, bf, N, K, 128));
     return launch_pair<256>(ta, tb, ep, M, N, K, st);
@@ -1293,23 +1233,27 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
   // (gated epilogues are the longest, and the single-buffered tall tile cannot hide them: 128-row tiles there)
   if (g_tm_override == 256 || (g_tm_override == 0 && g_bn_override == 0 && !gated && pick_tall(M, N, K)))
     tm = 256, bn = 256;
-  // cluster multicast of the W tile across two M tiles (measured neutral on GB300; kept selectable)
-  const int cl = g_cl_override == 2 ? 2 : 1;
   SR_TRY(encode_kmajor(&ta, A, bf, M, K, tm));
-  SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn / cl));
-  if (tm == 256) return cl == 2 ? launch_bn<256, 256, 2>(ta, tb, ep, M, N, K, st)
-                                : launch_bn<256, 256, 1>(ta, tb, ep, M, N, K, st);
-  if (cl == 2) {
-    if (bn == 64) return launch_bn<128, 64, 2>(ta, tb, ep, M, N, K, st);
-    if (bn == 128) return launch_bn<128, 128, 2>(ta, tb, ep, M, N, K, st);
-    return launch_bn<128, 256, 2>(ta, tb, ep, M, N, K, st);
-  }
-  if (bn == 64) return launch_bn<128, 64, 1>(ta, tb, ep, M, N, K, st);
-  if (bn == 128) return launch_bn<128, 128, 1>(ta, tb, ep, M, N, K, st);
-  return launch_bn<128, 256, 1>(ta, tb, ep, M, N, K, st);
+  SR_TRY(encode_kmajor(&tb, W, bf, N, K, bn));
+  if (tm == 256) return launch_bn<256, 256>(ta, tb, ep, M, N, K, st);
+  if (bn == 64) return launch_bn<128, 64>(ta, tb, ep, M, N, K, st);
+  if (bn == 128) return launch_bn<128, 128>(ta, tb, ep, M, N, K, st);
+  return launch_bn<128, 256>(ta, tb, ep, M, N, K, st);
 }
 
 // Device error word of the tensor-core GEMM (nonzero after a bounded wait expired).
 int* gemm_error_word() { return g_err; }
+
+// Free the split-K workspace kept for `st` on the current device (called when a context that used the
+// stream is destroyed; the stream must have no GEMM in flight).
+void gemm_release_workspace(cudaStream_t st) {
+  int dev;
+  if (cudaGetDevice(&dev) != cudaSuccess) return;
+  std::lock_guard<std::mutex> lk(g_ws_mu);
+  auto it = g_ws.find(std::make_pair(dev, st));
+  if (it == g_ws.end()) return;
+  if (it->second.first) cudaFree(it->second.first);
+  g_ws.erase(it);
+}
 
 }  // namespace sr
