@@ -298,13 +298,18 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
  * no counterpart; this is an interface convenience.  Instead of a per-call buffer, the split
  * partials (needed when a context exceeds 512 positions) use one fixed 8 MiB device array that
  * every GPU loading the library holds until exit; the call allocates nothing.
- *   max_len : an upper bound on lens[] (sizes the number of 512-position splits).
+ *   max_len : an upper bound on lens[]; it sizes the number of 512-position splits,
+ *             ceil(min(max_len, window or max_len) / 512).  No shared-prefix pass (shared_pos = 0).
  * Rejects, with SR_ERR_INVALID_ARG and a message, shapes needing more than 2^21 scratch floats
- * (b * n_heads * splits * (head_dim + 2)).  The first call on a device looks up the array's device
- * address (cudaGetSymbolAddress) with that device current; make that first call before any stream
- * capture.  All calls share the array and it keeps the last call's contents (every value a call
- * reads it has written itself, so nothing needs clearing); calls that overlap on the GPU, e.g. on
- * two streams, race on it. */
+ * (b * n_heads * splits * (head_dim + 2)).  lens[] is read on the device: a row whose length needs
+ * more splits than max_len gives is computed over its first `splits` splits only (nothing is read
+ * or written outside the array), a device flag records it, and the call returns SR_ERR_INVALID_ARG
+ * with `out` not valid.  To read that flag the call synchronises `stream` before it returns.  The
+ * first call on a device looks up the array's device address (cudaGetSymbolAddress) with that
+ * device current; make that first call before any stream capture.  All calls share the array and
+ * it keeps the last call's contents (every partial a call reads it has written itself, and the
+ * flag is cleared at the start of each call); calls that overlap on the GPU, e.g. on two streams,
+ * race on it. */
 sr_status sr_k_decode_attention_static(int dtype, const void* q, const void* pool, const int32_t* page_table,
                                        int pt_stride, const int32_t* orig_ids, const int32_t* lens, int b,
                                        int n_heads, int n_kv_heads, int head_dim, int window, int max_len, void* out,

@@ -25,12 +25,22 @@ namespace {
 
 constexpr int SPLIT = 512;  // KV positions per decode split
 
+// A row's split count, limited to the `slots` partial slots the launch provides per (row, head).  A
+// row needing more (its length exceeds the bound the launch was sized for) keeps only its first `slots`
+// splits, and `err` (when given) records the overrun, so no read or write leaves the row's slots.
+__device__ __forceinline__ int clamp_splits(int nsplit, int slots, int* err) {
+  if (nsplit <= slots) return nsplit;
+  if (err) atomicExch(err, 1);
+  return slots;
+}
+
 template <typename T, int DH, int G>
 __global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, const T* __restrict__ pool,
                                                      const int* __restrict__ pt, int pt_stride,
                                                      const int* __restrict__ slot_ids, const int* __restrict__ lens,
                                                      int Hkv, float scale_log2, int window, int max_splits,
-                                                     T* __restrict__ out, float* __restrict__ part) {
+                                                     T* __restrict__ out, float* __restrict__ part,
+                                                     int* __restrict__ err) {
   pdl_entry();
   constexpr int VE = 16 / sizeof(T);  // elements per 16-byte vector
   constexpr int TPT = DH / VE;        // threads per token
@@ -43,7 +53,7 @@ __global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, co
   const int Hq = Hkv * G;
   const int L = lens[s];
   const int t_lo = window > 0 ? max(0, L - window) : 0;
-  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  const int nsplit = clamp_splits((L - t_lo + SPLIT - 1) / SPLIT, max_splits, err);
   if (split >= nsplit) return;
   const int t_begin = t_lo + split * SPLIT, t_end = min(L, t_begin + SPLIT);
   const int tid = threadIdx.x, grp = tid / TPT, sub = tid % TPT, d0 = sub * VE;
@@ -140,12 +150,12 @@ __global__ void __launch_bounds__(128) k_decode_attn(const T* __restrict__ q, co
 // prefix and the position splits start at slot 1 (sbase = 1, suffix positions from t_min).
 template <typename T, int DH>
 __global__ void k_decode_combine(const float* __restrict__ part, const int* __restrict__ lens, int Hq, int window,
-                                 int max_splits, int t_min, int sbase, T* __restrict__ out) {
+                                 int max_splits, int t_min, int sbase, T* __restrict__ out, int* __restrict__ err) {
   pdl_entry();
   const int hq = blockIdx.x, s = blockIdx.y, d = threadIdx.x;
   const int L = lens[s];
   const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
-  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  const int nsplit = clamp_splits((L - t_lo + SPLIT - 1) / SPLIT, max_splits - sbase, err);
   if (nsplit <= 1 && (sbase == 0 || nsplit == 1)) return;  // written directly by the attention kernel
   const int total = sbase + nsplit;
   const float* pp = part + ((size_t)s * Hq + hq) * max_splits * (DH + 2);
@@ -246,7 +256,8 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
                                                         const int* __restrict__ slot_ids,
                                                         const int* __restrict__ lens, int Hkv, float scale_log2,
                                                         int window, int t_min, int sbase, int max_splits,
-                                                        T* __restrict__ out, float* __restrict__ part) {
+                                                        T* __restrict__ out, float* __restrict__ part,
+                                                        int* __restrict__ err) {
   pdl_entry();
   static_assert(G >= 1 && G <= 8 && DH % 16 == 0, "shape");
   constexpr int LDS = DH + 8;                  // padded smem row (elements): conflict-free ldmatrix
@@ -269,7 +280,7 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
   const int Hq = Hkv * G;
   const int L = lens[s];
   const int t_lo = max(t_min, window > 0 ? max(0, L - window) : 0);
-  const int nsplit = (L - t_lo + SPLIT - 1) / SPLIT;
+  const int nsplit = clamp_splits((L - t_lo + SPLIT - 1) / SPLIT, max_splits - sbase, err);
   if (split >= nsplit) return;
   const int t_begin = t_lo + split * SPLIT, t_end = min(L, t_begin + SPLIT);
   const int p_first = t_begin / PAGE, n_pages = (t_end - 1) / PAGE - p_first + 1;
@@ -855,7 +866,7 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
 template <typename T, int DH, int G>
 sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
                            const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
-                           int shared_pos, int max_len, cudaStream_t st) {
+                           int shared_pos, int max_len, cudaStream_t st, int* err) {
   // with a shared prefix: slot 0 of the partials is the prefix pass, position splits follow
   const int sbase = shared_pos > 0 ? 1 : 0;
   const int t_min = shared_pos;
@@ -890,16 +901,16 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
   if (max_len > 0 && span <= 8 * PAGE && max_splits - sbase == 1) {
     dim3 grid((Hkv + 3) / 4, b, 1);
     launch_k(k_decode_attn_tc<T, DH, G, 1>, grid, 128, smem, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens,
-             Hkv, scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
+             Hkv, scale_log2, window, t_min, sbase, max_splits, (T*)out, part, err);
   } else {
     dim3 grid(Hkv, b, max_splits - sbase);
     launch_k(k_decode_attn_tc<T, DH, G, 4>, grid, 128, smem, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens,
-             Hkv, scale_log2, window, t_min, sbase, max_splits, (T*)out, part);
+             Hkv, scale_log2, window, t_min, sbase, max_splits, (T*)out, part, err);
   }
   SR_LAUNCH();
   if (max_splits - sbase > 1) {  // some row has several position splits (a lone split merges the prefix itself)
     launch_k(k_decode_combine<T, DH>, dim3(Hkv * G, b), DH, 0, st, part, lens, Hkv * G, window, max_splits, t_min, sbase,
-                                                             (T*)out);
+             (T*)out, err);
     SR_LAUNCH();
   }
   return SR_OK;
@@ -908,15 +919,15 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
 template <typename T, int DH, int G>
 sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
                         const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
-                        cudaStream_t st) {
+                        cudaStream_t st, int* err) {
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid(Hkv, b, max_splits);
   launch_k(k_decode_attn<T, DH, G>, grid, 128, 0, st, (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, Hkv,
-                                                 scale_log2, window, max_splits, (T*)out, part);
+           scale_log2, window, max_splits, (T*)out, part, err);
   SR_LAUNCH();
   if (max_splits > 1) {
     launch_k(k_decode_combine<T, DH>, dim3(Hkv * G, b), DH, 0, st, part, lens, Hkv * G, window, max_splits, 0, 0,
-                                                             (T*)out);
+             (T*)out, err);
     SR_LAUNCH();
   }
   return SR_OK;
@@ -956,7 +967,7 @@ size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits) {
 sr_status launch_decode_attention(int et, const void* q, const void* pool_layer, const int* pt, int pt_stride,
                                   const int* ids, const int* lens, int b, int Hq, int Hkv, int dh, int window,
                                   void* out, float* part, int max_splits, cudaStream_t st, int shared_pos,
-                                  int max_len) {
+                                  int max_len, int* err) {
   if (b == 0) return SR_OK;
   const int G = Hq / Hkv;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "decode attention: n_heads %% n_kv_heads != 0");
@@ -964,11 +975,11 @@ sr_status launch_decode_attention(int et, const void* q, const void* pool_layer,
 #define SR_DEC(T, D, GG)                                                                                          \
   if (dh == D && G == GG)                                                                                         \
     return decode_attn_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
-                                   st);
+                                   st, err);
 #define SR_DECT(T, D, GG)                                                                                          \
   if (dh == D && G == GG)                                                                                            \
     return decode_attn_tc_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
-                                      shared_pos, max_len, st);
+                                      shared_pos, max_len, st, err);
   if (et == SR_DT_F16) {
     SR_DECT(f16, 128, 4) SR_DECT(f16, 128, 1) SR_DECT(f16, 128, 2) SR_DECT(f16, 128, 8)
     SR_DECT(f16, 64, 1) SR_DECT(f16, 64, 4) SR_DECT(f16, 32, 1)
@@ -1039,33 +1050,41 @@ sr_status launch_prefill_attention(int et, const void* q, const void* k, const v
 // budget (an inference server that reserves all of the GPU's memory up front), allocator-free
 // embeddings, or callers holding locks under which an allocation could block.  For them the split
 // partials of decode attention live in this fixed device array instead of a buffer allocated per
-// call.  Every GPU that loads the library holds the array (8 MiB) until the process exits.
+// call, next to one int the kernels set when a row is longer than the caller's bound.  Every GPU
+// that loads the library holds the array (8 MiB) until the process exits.
 // -------------------------------------------------------------------------------------------------
 namespace sr {
 namespace {
 
 constexpr size_t kStaticPartFloats = (size_t)1 << 21;  // 8 MiB of fp32 split partials
 static __device__ __align__(256) float g_static_part[kStaticPartFloats];
+static __device__ __align__(256) int g_static_err;      // 1 after a row needed more splits than max_len allows
 
 constexpr int kMaxDevices = 64;
 std::mutex g_static_mu;
-float* g_static_ptr[kMaxDevices] = {};  // device address of g_static_part, per device ordinal
+struct StaticScratch {
+  float* part = nullptr;  // device address of g_static_part
+  int* err = nullptr;     // device address of g_static_err
+};
+StaticScratch g_static[kMaxDevices];  // per device ordinal
 
-// In host code `g_static_part` names a host-side stand-in, not device memory, so its device
-// address is looked up once per device (with that device current) and cached.
-sr_status static_part_ptr(float** out) {
+// In host code `g_static_part` and `g_static_err` name host-side stand-ins, not device memory, so
+// their device addresses are looked up once per device (with that device current) and cached.
+sr_status static_scratch(StaticScratch* out) {
   int dev = 0;
   SR_CUDA(cudaGetDevice(&dev));
   if (dev < 0 || dev >= kMaxDevices) return set_err(SR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
   std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_ptr[dev]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_part);
-    if (e != cudaSuccess)
-      return set_err(SR_ERR_CUDA, "cudaGetSymbolAddress(static decode-attention scratch): %s", cudaGetErrorString(e));
-    g_static_ptr[dev] = static_cast<float*>(p);
+  if (!g_static[dev].part) {
+    void *p = nullptr, *e = nullptr;
+    cudaError_t r = cudaGetSymbolAddress(&p, g_static_part);
+    if (r == cudaSuccess) r = cudaGetSymbolAddress(&e, g_static_err);
+    if (r != cudaSuccess)
+      return set_err(SR_ERR_CUDA, "cudaGetSymbolAddress(static decode-attention scratch): %s", cudaGetErrorString(r));
+    g_static[dev].part = static_cast<float*>(p);
+    g_static[dev].err = static_cast<int*>(e);
   }
-  *out = g_static_ptr[dev];
+  *out = g_static[dev];
   return SR_OK;
 }
 
@@ -1082,16 +1101,30 @@ extern "C" sr_status sr_k_decode_attention_static(int dtype, const void* q, cons
   if (b < 0 || n_kv_heads < 1 || n_heads < 1 || head_dim < 1 || max_len < 1)
     return set_err(SR_ERR_INVALID_ARG, "sr_k_decode_attention_static: bad shape");
   const int splits = decode_attention_max_splits(window > 0 ? std::min(max_len, window) : max_len);
-  float* part = nullptr;
-  if (splits > 1) {
-    const size_t need = decode_attention_part_floats(b, n_heads, head_dim, splits);
-    if (need > kStaticPartFloats)
-      return set_err(SR_ERR_INVALID_ARG,
-                     "sr_k_decode_attention_static: %zu scratch floats needed (b=%d, heads=%d, head_dim=%d, %d "
-                     "splits of %d positions) but the static scratch holds %zu",
-                     need, b, n_heads, head_dim, splits, SPLIT, kStaticPartFloats);
-    SR_TRY(static_part_ptr(&part));
-  }
-  return launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
-                                 head_dim, window, out, part, splits, static_cast<cudaStream_t>(stream));
+  const size_t need = splits > 1 ? decode_attention_part_floats(b, n_heads, head_dim, splits) : 0;
+  if (need > kStaticPartFloats)
+    return set_err(SR_ERR_INVALID_ARG,
+                   "sr_k_decode_attention_static: %zu scratch floats needed (b=%d, heads=%d, head_dim=%d, %d "
+                   "splits of %d positions) but the static scratch holds %zu",
+                   need, b, n_heads, head_dim, splits, SPLIT, kStaticPartFloats);
+  if (b == 0) return SR_OK;
+  StaticScratch sc;
+  SR_TRY(static_scratch(&sc));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // the error word keeps the last call's value: clear it before the kernels run
+  SR_CUDA(cudaMemsetAsync(sc.err, 0, sizeof(int), st));
+  SR_TRY(launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
+                                 head_dim, window, out, splits > 1 ? sc.part : nullptr, splits, st, 0, max_len,
+                                 sc.err));
+  // lens[] lives on the device, so whether every length was within max_len is known only once the
+  // kernels ran: read their flag back (this synchronises `stream`)
+  int h_err = 0;
+  SR_CUDA(cudaMemcpyAsync(&h_err, sc.err, sizeof(int), cudaMemcpyDeviceToHost, st));
+  SR_CUDA(cudaStreamSynchronize(st));
+  if (h_err)
+    return set_err(SR_ERR_INVALID_ARG,
+                   "sr_k_decode_attention_static: a length in lens[] exceeds max_len = %d by more than its last "
+                   "512-position split; the rows concerned kept only their first %d split(s) and `out` is not valid",
+                   max_len, splits);
+  return SR_OK;
 }

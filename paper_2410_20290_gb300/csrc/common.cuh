@@ -198,7 +198,8 @@ sr_status launch_sample(const float* logits, long long ld, int b, int V, const i
 sr_status launch_decode_attention(int dtype, const void* q, const void* pool_layer, const int* page_table,
                                   int pt_stride, const int* slot_ids, const int* lens, int b, int Hq, int Hkv, int dh,
                                   int window, void* out, float* part, int max_splits, cudaStream_t st,
-                                  int shared_pos = 0, int max_len = 0);  // max_len > 0: longest lens[] (launch shape)
+                                  int shared_pos = 0, int max_len = 0,  // max_len > 0: longest lens[] (launch shape)
+                                  int* err = nullptr);  // set to 1 when a row needs more splits than max_splits
 int decode_attention_max_splits(int max_len);
 int decode_attention_slots(int max_len, int window, int shared_pos);
 size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits);
