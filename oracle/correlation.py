@@ -3,9 +3,12 @@
 Appendix B measures how well the reward of a partial response Y^{<=tau} predicts the reward of the
 complete response: for Best-of-N trajectories, the partial reward at each decision point tau
 (tau_k = min(tau, len(Y_k)), Eq. partial.reward.set) against the final reward, summarised by the
-Pearson correlation and Kendall's rank correlation.  Kendall's tau-b (ties in either vector
-corrected) is used.  Both statistics are written from their definitions; pinned against scipy and
-brute force in tests/test_oracle_correlation.py.  Test infrastructure only.
+Pearson correlation and Kendall's rank correlation.  Appendix B defines Kendall's statistic as
+R_Kendall = 2 / (N (N - 1)) sum_{i<j} sgn(x_i - x_j) sgn(y_i - y_j), the plain tau-a (a tied pair
+contributes 0 and the denominator counts every pair); that is what `kendall_tau_a` computes.  The
+tie-corrected tau-b is kept as an extra figure.  Every statistic is written from its definition;
+pinned against scipy, hand-computed vectors and brute force in tests/test_oracle_correlation.py.
+Test infrastructure only.
 """
 from typing import Sequence
 
@@ -20,6 +23,20 @@ def pearson(x, y) -> float:
     dx, dy = x - x.mean(), y - y.mean()
     den = np.sqrt(np.sum(dx * dx) * np.sum(dy * dy))
     return float(np.sum(dx * dy) / den) if den > 0 else float("nan")
+
+
+def kendall_tau_a(x, y) -> float:
+    """Appendix B: 2 / (n (n - 1)) sum_{i<j} sgn(x_i - x_j) sgn(y_i - y_j)."""
+    x = np.asarray(x, np.float64)
+    y = np.asarray(y, np.float64)
+    n = len(x)
+    if n < 2:
+        return float("nan")
+    total = 0
+    for i in range(n):
+        for j in range(i + 1, n):
+            total += int(np.sign(x[i] - x[j])) * int(np.sign(y[i] - y[j]))
+    return 2.0 * total / (n * (n - 1))
 
 
 def kendall_tau_b(x, y) -> float:
@@ -46,8 +63,10 @@ def kendall_tau_b(x, y) -> float:
 
 def partial_final(gen, rm, prompt, N: int, taus: Sequence[int], max_new: int, temperature: float, eos_bias: float,
                   eos_id: int, seed: int):
-    """Best-of-N responses; partial rewards at each tau, final rewards, and per-tau (Pearson, Kendall tau-b)."""
+    """Best-of-N responses; partial rewards at each tau, final rewards, and per-tau (Pearson, Kendall tau-a of
+    Appendix B, Kendall tau-b)."""
     _, _, _, seqs, final = best_of_n(gen, rm, prompt, N, max_new, temperature, eos_bias, eos_id, seed)
     partial = {t: score_sequences(rm, prompt, [y[:min(t, len(y))] for y in seqs]) for t in taus}
-    stats = {t: (pearson(partial[t], final), kendall_tau_b(partial[t], final)) for t in taus}
+    stats = {t: (pearson(partial[t], final), kendall_tau_a(partial[t], final), kendall_tau_b(partial[t], final))
+             for t in taus}
     return partial, final, stats

@@ -3,7 +3,6 @@ import numpy as np
 import pytest
 
 torch = pytest.importorskip("torch")
-pytest.importorskip("scipy")
 
 import sr_inputs as si
 from oracle import correlation as oc
@@ -32,5 +31,7 @@ def test_tiny_partial_final_correlation_matches_oracle():
     for t in taus:
         np.testing.assert_allclose(part[t], opart[t], rtol=0, atol=tol)
         assert abs(stats[t][0] - ostats[t][0]) <= 1e-2
+        # each pair whose order flips within the reward tolerance moves tau-a by 2 / (N (N - 1))
         assert abs(stats[t][1] - ostats[t][1]) <= 2.0 / (w.N * (w.N - 1) / 2) + 1e-9
+        assert abs(stats[t][2] - ostats[t][2]) <= 3.0 / (w.N * (w.N - 1) / 2) + 1e-9
     assert stats[taus[-1]][0] == pytest.approx(1.0)
