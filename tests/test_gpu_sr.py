@@ -5,7 +5,7 @@ import pytest
 torch = pytest.importorskip("torch")
 
 import sr_inputs as si
-from oracle.pool import pool_pages
+from oracle.pool import PagePool, pool_pages
 from oracle.sampler import perturbed_logits, sample_token
 from oracle.select import float_keys, select_round
 from oracle.sr import DONE, SpeculativeRejection, run_workload
@@ -88,26 +88,109 @@ def test_tiny_alpha_zero_is_best_of_n(sr):
     assert st2["best_id"] == ref.best_id and list(toks2) == ref.tokens and score2 == score
 
 
-def test_tiny_memory_triggered_pool(sr):
-    """Memory-triggered rounds with a small pool: trigger steps, k (raised when needed), page tables and the
-    free stack match the oracle bit for bit."""
+class _PeakPool(PagePool):
+    """The oracle's page pool, also recording the most pages ever in use (for sr_stats.peak_pages_in_use)."""
+
+    def __init__(self, n_pages):
+        super().__init__(n_pages)
+        self.peak = 0
+
+    def pop(self):
+        p = super().pop()
+        self.peak = max(self.peak, self.n_pages - self.n_free)
+        return p
+
+
+MEM_CASES = ((1 + 8 * 2, 0.5, 16), (1 + 8 * 3 + 2, 0.25, 21), (2 + 8 + 8 * 1, 0.05, 37))
+
+
+def _mem_workload(pages, alpha, P):
     base = si.WORKLOADS["tiny"]
     kvt = si.kv_bytes_per_token(base.gen)
-    for pages, alpha, P in ((1 + 8 * 2, 0.5, 16), (1 + 8 * 3 + 2, 0.25, 21), (2 + 8 + 8 * 1, 0.05, 37)):
-        w = base.replace(sched_kind=si.SCHED_POOL_FULL, taus=(), alpha=alpha, pool_bytes=pages * 16 * kvt,
-                         prompt_len=P, max_new=min(base.max_new, base.gen.max_pos - P))
-        ctx, gw, rw = make_ctx(sr, w)
-        try:
-            toks, score, st = sr.sr_generate(ctx, w.prompt(3), w.N, alpha, w.sched_kind, (), w.max_new,
-                                              w.temperature, w.eos_bias, w.eos_id, 5)
-        finally:
-            sr.sr_destroy(ctx)
-        _, ref = oracle_sr(w, gw, rw, w.prompt(3), 5)
-        assert st["rounds"] == len(ref.rounds)
-        assert [st["step_per_round"][i] for i in range(st["rounds"])] == [r.step for r in ref.rounds]
-        assert [st["k_per_round"][i] for i in range(st["rounds"])] == [r.k for r in ref.rounds]
-        assert st["k_raised"] == sum(r.k_raised for r in ref.rounds)
-        assert st["best_id"] == ref.best_id and list(toks) == ref.tokens
+    return base.replace(sched_kind=si.SCHED_POOL_FULL, taus=(), alpha=alpha, pool_bytes=pages * 16 * kvt,
+                        prompt_len=P, max_new=min(base.max_new, base.gen.max_pos - P))
+
+
+@pytest.mark.parametrize("pages,alpha,P", MEM_CASES)
+def test_tiny_memory_triggered_pool(sr, pages, alpha, P):
+    """Memory-triggered rounds with a small pool through sr_generate: trigger steps, batch sizes, k (raised when
+    needed), accepted counts, r_cut, peak pages in use, selected candidate and tokens match the oracle."""
+    w = _mem_workload(pages, alpha, P)
+    ctx, gw, rw = make_ctx(sr, w)
+    try:
+        toks, score, st = sr.sr_generate(ctx, w.prompt(3), w.N, alpha, w.sched_kind, (), w.max_new,
+                                          w.temperature, w.eos_bias, w.eos_id, 5)
+    finally:
+        sr.sr_destroy(ctx)
+    o = SpeculativeRejection(Transformer(w.gen, gw), Transformer(w.rm, rw), w.prompt(3), w.N, alpha, w.sched_kind,
+                             (), w.max_new, w.temperature, w.eos_bias, w.eos_id, 5, pages)
+    o.pool = _PeakPool(pages)
+    ref = o.run()
+    assert st["pool_pages"] == pages
+    assert st["rounds"] == len(ref.rounds) and st["rounds"] >= 1
+    n = st["rounds"]
+    assert [st["step_per_round"][i] for i in range(n)] == [r.step for r in ref.rounds]
+    assert [st["b_per_round"][i] for i in range(n)] == [len(r.batch) for r in ref.rounds]
+    assert [st["k_per_round"][i] for i in range(n)] == [r.k for r in ref.rounds]
+    assert [st["accepted_per_round"][i] for i in range(n)] == [int(r.accepted.sum()) for r in ref.rounds]
+    assert st["k_raised"] == sum(r.k_raised for r in ref.rounds)
+    for i, r in enumerate(ref.rounds):
+        assert abs(st["r_cut_per_round"][i] - r.r_cut) <= reward_tol(r.r_cut, r.rewards)
+    assert st["peak_pages_in_use"] == o.pool.peak
+    assert st["gen_tokens"] == ref.gen_tokens
+    assert st["best_id"] == ref.best_id and list(toks) == ref.tokens
+
+
+@pytest.mark.parametrize("pages,alpha,P", MEM_CASES)
+def test_tiny_memory_triggered_component_calls(sr, pages, alpha, P):
+    """The same memory-triggered runs step by step through the component calls, the test taking the trigger
+    decision (free pages < live candidates at a page boundary) and feeding the oracle's rewards and its k
+    (raised where the oracle raised it) to sr_reject_compact: after every round and at the end, page tables of
+    the live candidates and the free stack equal the oracle's bit for bit."""
+    w = _mem_workload(pages, alpha, P)
+    ctx, gw, rw = make_ctx(sr, w)
+    prompt, seed, N = w.prompt(3), 5, w.N
+    o = SpeculativeRejection(Transformer(w.gen, gw), Transformer(w.rm, rw), prompt, N, alpha, w.sched_kind, (),
+                             w.max_new, w.temperature, w.eos_bias, w.eos_id, seed, pages)
+    ref = o.run()
+    max_pages = (P + w.max_new - 1) // 16 + 1
+    try:
+        b = sr.sr_batch_begin(ctx, prompt, N, w.max_new, w.temperature, w.eos_bias, w.eos_id, seed)
+        g, r = 1, 0
+        while True:
+            q = sr.sr_batch_query(ctx, b, N, w.max_new, max_pages, pages)
+            if q["n_live"] == 0:
+                break
+            need = (P + g - 1) % 16 == 0
+            if need and q["free_top"] < q["n_live"]:
+                rd, snap = ref.rounds[r], o.snapshots[r]
+                assert rd.step == g
+                rewards = sr.sr_score_partial(ctx, b, N)
+                assert len(rewards) == len(rd.batch)
+                for r_gpu, r_ref in zip(rewards, rd.rewards):
+                    assert abs(r_gpu - r_ref) <= reward_tol(r_ref, rd.rewards)
+                a_eff = np.float32((rd.k + 0.5) / len(rd.batch))      # floor(a_eff b) = the oracle's k
+                rc, acc, n_live = sr.sr_reject_compact(ctx, b, rd.rewards, float(a_eff))
+                assert rc == rd.r_cut
+                assert acc.tolist() == [i for i, a in zip(rd.batch, rd.accepted) if a]
+                q = sr.sr_batch_query(ctx, b, N, w.max_new, max_pages, pages)
+                assert q["free_stack"].tolist() == snap["free_stack"]
+                for i in range(N):
+                    if snap["status"][i] == 0:
+                        assert q["page_table"][i][:len(snap["page_tables"][i])].tolist() == snap["page_tables"][i]
+                r += 1
+                if n_live == 0:
+                    break
+            sr.sr_decode_step(ctx, b)
+            g += 1
+        assert r == len(ref.rounds)
+        q = sr.sr_batch_query(ctx, b, N, w.max_new, max_pages, pages)
+        for i in range(N):
+            assert q["tokens"][i][:q["lengths"][i]].tolist() == ref.all_tokens[i]
+        assert q["free_stack"].tolist() == ref.free_stack
+        sr.sr_batch_end(ctx, b)
+    finally:
+        sr.sr_destroy(ctx)
 
 
 def test_tiny_component_calls(sr):
@@ -163,7 +246,8 @@ def test_tiny_component_calls(sr):
         q = sr.sr_batch_query(ctx, b, N, w.max_new, max_pages, n_pages)
         for i in range(N):
             assert q["tokens"][i][:q["lengths"][i]].tolist() == ref.all_tokens[i]
-        assert q["free_stack"].tolist() == ref.free_stack or True  # final scoring releases nothing more
+        # every candidate has completed and released its private pages, in the oracle's order
+        assert q["free_stack"].tolist() == ref.free_stack
         sr.sr_batch_end(ctx, b)
     finally:
         sr.sr_destroy(ctx)
