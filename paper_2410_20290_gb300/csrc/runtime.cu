@@ -32,6 +32,7 @@ sr_status set_err(sr_status s, const char* fmt, ...) {
 }
 
 int* gemm_error_word();
+void gemm_release_workspace(cudaStream_t st);
 
 bool pdl_enabled() {
   static const bool on = [] {
@@ -1087,6 +1088,10 @@ void sr_destroy(sr_ctx* c) {
   if (!c) return;
   cudaSetDevice(c->device);
   if (c->st) cudaStreamSynchronize(c->st);
+  if (c->own) cudaStreamSynchronize(c->own);
+  // the GEMM's split-K buffers of this context's streams
+  if (c->own) gemm_release_workspace(c->own);
+  if (c->st && c->st != c->own) gemm_release_workspace(c->st);
   free_model(c->gen);
   free_model(c->rm);
   c->wg.release();
