@@ -116,7 +116,8 @@ typedef struct {
   int best_id;                            /* candidate id k* of the returned response */
   int waves;                              /* pool-sized Best-of-N waves (alpha = 0 with POOL_FULL), else 1 */
   long long gen_tokens;                   /* tokens sampled from the generator */
-  long long rm_tokens;                    /* positions run through the reward model (prompt once + partials) */
+  long long rm_tokens;                    /* positions run through the reward model: the prompt once, then every
+                                             scored response position not read from the reward-model cache */
   long long decode_steps;                 /* batched decode steps */
   int pool_pages;                         /* pages in the KV pool */
   int peak_pages_in_use;
@@ -133,6 +134,8 @@ typedef struct {
   long long kern_timed[SR_KC_N];    /* timed launches */
   double kern_timed_flops[SR_KC_N];
   double kern_timed_bytes[SR_KC_N];
+  long long rm_tokens_cached;  /* scored response positions whose reward-model K/V came from the cache
+                                  (sr_set_rm_cache) instead of being run again */
 } sr_stats;
 
 typedef struct sr_ctx sr_ctx;
@@ -179,6 +182,20 @@ sr_status sr_auto_b_init(const sr_model_desc* gen, size_t kv_pool_bytes, int P, 
  * The kind is read when a batch starts (sr_generate, sr_batch_begin); errors: SR_ERR_INVALID_ARG. */
 enum { SR_REWARD_MODEL = 0, SR_REWARD_LOGPROB = 1 };
 sr_status sr_set_reward(sr_ctx* ctx, int kind);
+/* Reward-model KV kept across rejection rounds.  A partial reward s(X ++ Y^{<=tau}) (Eq.
+ * partial.reward.set) needs the reward model's keys and values of every position before the last; the
+ * paper re-runs them at every round and at the final score, the cost Section 1 calls quadratic.  With
+ * `bytes` > 0 the library keeps, in a second paged pool of floor(bytes / (16 x the reward model's KV bytes
+ * per position)) pages, each candidate's reward-model K/V of the response positions it has scored; a later
+ * round, or the final score of a survivor, runs only the positions added since and attends to the cached
+ * ones.  At a round, the batch's new positions go into the pool for every candidate (ascending id) whose
+ * pages the free pool can still give; the others are scored in full as without the cache.  Rejected and
+ * finished candidates' pages return to the pool when the next scoring starts.  Results agree with full
+ * rescoring up to floating-point summation order.  0 (the default) turns it off.  Read when a batch starts
+ * (sr_generate, sr_batch_begin); a context holds the pool until sr_destroy or a call with bytes = 0.
+ * The prompt's reward-model KV is always computed once per batch.  Errors: SR_ERR_INVALID_ARG (null ctx);
+ * SR_ERR_OOM at the next sr_generate / sr_batch_begin when the pool cannot be allocated. */
+sr_status sr_set_rm_cache(sr_ctx* ctx, size_t bytes);
 /* Per-kernel-class CUDA-event timing: 0 off; k >= 1 times one launch in k of each class (1: every
    launch; each timed launch adds two event records to the stream) and counts all of them.  Results
    land in sr_stats.kern_*.  Errors: SR_ERR_INVALID_ARG (null context, k < 0). */

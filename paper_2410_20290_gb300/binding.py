@@ -55,7 +55,7 @@ class sr_stats(ctypes.Structure):
                 ("kern_ms", ctypes.c_double * SR_KC_N), ("kern_launches", ctypes.c_longlong * SR_KC_N),
                 ("kern_flops", ctypes.c_double * SR_KC_N), ("kern_bytes", ctypes.c_double * SR_KC_N),
                 ("kern_timed", ctypes.c_longlong * SR_KC_N), ("kern_timed_flops", ctypes.c_double * SR_KC_N),
-                ("kern_timed_bytes", ctypes.c_double * SR_KC_N)]
+                ("kern_timed_bytes", ctypes.c_double * SR_KC_N), ("rm_tokens_cached", ctypes.c_longlong)]
 
     def as_dict(self) -> dict:
         r = self.rounds
@@ -92,6 +92,7 @@ _SIG = {
     "sr_batch_end": [_P, _P],
     "sr_k_sample": [_P, ctypes.c_longlong, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P, _P],
     "sr_set_reward": [_P, _I],
+    "sr_set_rm_cache": [_P, ctypes.c_size_t],
     "sr_auto_b_init": [_P, ctypes.c_size_t, _I, _I, _I, _P],
     "sr_k_rcut": [_P, _I, _F, _I, _P, _P, _P],
     "sr_k_gemm": [_I, _P, _P, _P, _I, _I, _I, _I, _P],
@@ -191,6 +192,11 @@ def sr_auto_b_init(gen, kv_pool_bytes: int, P: int, tau_min: int, n_max: int) ->
         return 0
     _check(st)
     return n.value
+
+
+def sr_set_rm_cache(ctx, nbytes: int):
+    """Keep the reward model's KV across rounds in a pool of nbytes (0: off)."""
+    _check(LIB.sr_set_rm_cache(ctx, int(nbytes)))
 
 
 def sr_set_reward(ctx, kind: int):

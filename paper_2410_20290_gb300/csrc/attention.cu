@@ -510,7 +510,8 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
                                                       const int* __restrict__ seq_off,
                                                       const int* __restrict__ tile_seq,
                                                       const int* __restrict__ tile_q0, int pos0, int Hq, int Hkv,
-                                                      float scale_log2, int window, T* __restrict__ out) {
+                                                      float scale_log2, int window, T* __restrict__ out,
+                                                      CachedKeys ck) {
   pdl_entry();
   constexpr int LD = DH + 8, LDV = DV + 8;
   extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -537,36 +538,63 @@ __global__ void __launch_bounds__(128) k_prefill_attn(const T* __restrict__ q, c
 #pragma unroll
   for (int i = 0; i < DV / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  // cached keys of this sequence (positions pos0 .. pos0 + ncache - 1, paged); its own rows follow them
+  const int ncache = ck.pool ? ck.seq_cached[j] : 0;
+  const int* cpt = ck.pool ? ck.page_table + (size_t)ck.seq_cand[j] * ck.pt_stride : nullptr;
+  const int opos0 = pos0 + ncache;      // position of own row 0
   const int qi_a = q0 + warp * 16 + g;  // query index within the sequence (rows g and g + 8)
-  const int qpos[2] = {pos0 + qi_a, pos0 + qi_a + 8};
-  const int qpos_min = pos0 + q0;
-  const int qpos_max = pos0 + min(nrows, q0 + BQ) - 1;
+  const int qpos[2] = {opos0 + qi_a, opos0 + qi_a + 8};
+  const int qpos_min = opos0 + q0;
+  const int qpos_max = opos0 + min(nrows, q0 + BQ) - 1;
 
   const int nb_pre = (npre + BKV - 1) / BKV;
+  const int nb_c = (ncache + BKV - 1) / BKV;
   const int own_keys = min(nrows, q0 + BQ);
   const int nb_own = (own_keys + BKV - 1) / BKV;
+  const size_t cpage = (size_t)2 * Hkv * PAGE * DH;  // elements per cached page (K and V of every kv head)
 
-  for (int kb = 0; kb < nb_pre + nb_own; ++kb) {
-    const bool is_pre = kb < nb_pre;
-    const int kbase = is_pre ? kb * BKV : (kb - nb_pre) * BKV;   // key index within its segment
-    const int kcount = is_pre ? min(BKV, npre - kbase) : min(BKV, own_keys - kbase);
-    const int kpos0 = is_pre ? kbase : pos0 + kbase;
+  for (int kb = 0; kb < nb_pre + nb_c + nb_own; ++kb) {
+    const int seg = kb < nb_pre ? 0 : (kb < nb_pre + nb_c ? 1 : 2);  // prefix, cached, own
+    const int kbase = seg == 0 ? kb * BKV : (seg == 1 ? (kb - nb_pre) * BKV : (kb - nb_pre - nb_c) * BKV);
+    const int kcount = min(BKV, (seg == 0 ? npre : (seg == 1 ? ncache : own_keys)) - kbase);
+    const int kpos0 = seg == 0 ? kbase : (seg == 1 ? pos0 + kbase : opos0 + kbase);
     if (window > 0 && kpos0 + kcount - 1 <= qpos_min - window) continue;  // whole block left of every window
     if (kpos0 > qpos_max) continue;
     __syncthreads();  // previous block's smem reads are done
-    const T* ksrc = is_pre ? kpre : k + (size_t)r0 * kstride;
-    const T* vsrc = is_pre ? vpre : v + (size_t)r0 * kstride;
-    for (int c = tid; c < BKV * (DH / 8); c += 128) {
-      const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
-      const bool ok = row < kcount;
-      const T* src = ok ? ksrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + col : ksrc;
-      cp_async16(sK + row * LD + col, src, ok);
-    }
-    for (int c = tid; c < BKV * (DV / 8); c += 128) {
-      const int row = c / (DV / 8), col = (c % (DV / 8)) * 8;
-      const bool ok = row < kcount;
-      const T* src = ok ? vsrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + dvo + col : vsrc;
-      cp_async16(sV + row * LDV + col, src, ok);
+    if (seg == 1) {
+      const T* cpool = reinterpret_cast<const T*>(ck.pool);
+      for (int c = tid; c < BKV * (DH / 8); c += 128) {
+        const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+        const bool ok = row < kcount;
+        const int t = kbase + row;
+        const T* src = ok ? cpool + (size_t)cpt[t / PAGE] * cpage + ((size_t)hk * PAGE + t % PAGE) * DH + col : cpool;
+        cp_async16(sK + row * LD + col, src, ok);
+      }
+      for (int c = tid; c < BKV * (DV / 8); c += 128) {
+        const int row = c / (DV / 8), col = (c % (DV / 8)) * 8;
+        const bool ok = row < kcount;
+        const int t = kbase + row;
+        const T* src = ok ? cpool + (size_t)cpt[t / PAGE] * cpage + ((size_t)(Hkv + hk) * PAGE + t % PAGE) * DH + dvo +
+                                col
+                          : cpool;
+        cp_async16(sV + row * LDV + col, src, ok);
+      }
+    } else {
+      const bool is_pre = seg == 0;
+      const T* ksrc = is_pre ? kpre : k + (size_t)r0 * kstride;
+      const T* vsrc = is_pre ? vpre : v + (size_t)r0 * kstride;
+      for (int c = tid; c < BKV * (DH / 8); c += 128) {
+        const int row = c / (DH / 8), col = (c % (DH / 8)) * 8;
+        const bool ok = row < kcount;
+        const T* src = ok ? ksrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + col : ksrc;
+        cp_async16(sK + row * LD + col, src, ok);
+      }
+      for (int c = tid; c < BKV * (DV / 8); c += 128) {
+        const int row = c / (DV / 8), col = (c % (DV / 8)) * 8;
+        const bool ok = row < kcount;
+        const T* src = ok ? vsrc + (size_t)(kbase + row) * kstride + (size_t)hk * DH + dvo + col : vsrc;
+        cp_async16(sV + row * LDV + col, src, ok);
+      }
     }
     cp_async_wait_all();
     __syncthreads();
@@ -817,21 +845,33 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
                                    const float* __restrict__ v, const float* __restrict__ kpre,
                                    const float* __restrict__ vpre, int npre, const int* __restrict__ seq_off,
                                    int n_seq, int pos0, int Hq, int Hkv, int dh, float scale, int window,
-                                   float* __restrict__ out) {
+                                   float* __restrict__ out, CachedKeys ck) {
   pdl_entry();
   extern __shared__ float sc[];
   __shared__ float red[32];
   const int r = blockIdx.x, hq = blockIdx.y, hk = hq / (Hq / Hkv);
   int j = 0;
   while (j + 1 < n_seq && seq_off[j + 1] <= r) ++j;
-  const int r0 = seq_off[j], qi = r - r0, qpos = pos0 + qi;
-  const int nk = npre + qi + 1;
+  // keys: npre prefix keys, ncache cached keys (paged, positions pos0 ..), then the sequence's own rows
+  const int ncache = ck.pool ? ck.seq_cached[j] : 0;
+  const int* cpt = ck.pool ? ck.page_table + (size_t)ck.seq_cand[j] * ck.pt_stride : nullptr;
+  const float* cpool = reinterpret_cast<const float*>(ck.pool);
+  const size_t cpage = (size_t)2 * Hkv * PAGE * dh;
+  const int r0 = seq_off[j], qi = r - r0, qpos = pos0 + ncache + qi;
+  const int nk = npre + ncache + qi + 1;
+  auto key_row = [&](int t, int which) -> const float* {  // which 0: K, 1: V
+    if (t < npre) return (which ? vpre : kpre) + ((size_t)t * Hkv + hk) * dh;
+    if (t < npre + ncache) {
+      const int c = t - npre;
+      return cpool + (size_t)cpt[c / PAGE] * cpage + ((size_t)(which * Hkv + hk) * PAGE + c % PAGE) * dh;
+    }
+    return (which ? v : k) + ((size_t)(r0 + t - npre - ncache) * Hkv + hk) * dh;
+  };
   const float* qr = q + ((size_t)r * Hq + hq) * dh;
   float mx = -INFINITY;
   for (int t = threadIdx.x; t < nk; t += blockDim.x) {
-    const bool pre = t < npre;
-    const int kpos = pre ? t : pos0 + (t - npre);
-    const float* kr = pre ? kpre + ((size_t)t * Hkv + hk) * dh : k + ((size_t)(r0 + t - npre) * Hkv + hk) * dh;
+    const int kpos = t < npre ? t : pos0 + (t - npre);
+    const float* kr = key_row(t, 0);
     float s = 0.f;
     for (int d = 0; d < dh; ++d) s = fmaf(qr[d], kr[d], s);
     s *= scale;
@@ -854,11 +894,7 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
   sum = block_sum(sum, red);
   for (int d = threadIdx.x; d < dh; d += blockDim.x) {
     float o = 0.f;
-    for (int t = 0; t < nk; ++t) {
-      const bool pre = t < npre;
-      const float* vr = pre ? vpre + ((size_t)t * Hkv + hk) * dh : v + ((size_t)(r0 + t - npre) * Hkv + hk) * dh;
-      o = fmaf(sc[t], vr[d], o);
-    }
+    for (int t = 0; t < nk; ++t) o = fmaf(sc[t], key_row(t, 1)[d], o);
     out[((size_t)r * Hq + hq) * dh + d] = o / sum;
   }
 }
@@ -936,7 +972,7 @@ sr_status decode_attn_t(const void* q, const void* pool, const int* pt, int pt_s
 template <typename T, int DH, int DV>
 sr_status prefill_t(const void* q, const void* k, const void* v, const void* kpre, const void* vpre, int npre,
                     const int* seq_off, const int* tile_seq, const int* tile_q0, int n_tiles, int pos0, int Hq,
-                    int Hkv, int window, void* out, cudaStream_t st) {
+                    int Hkv, int window, void* out, cudaStream_t st, CachedKeys ck) {
   const size_t smem = (size_t)(BQ * (DH + 8) + BKV * (DH + 8) + BKV * (DV + 8)) * sizeof(T);
   static bool attr_set = false;
   if (!attr_set) {
@@ -946,8 +982,7 @@ sr_status prefill_t(const void* q, const void* k, const void* v, const void* kpr
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid(n_tiles, Hq, DH / DV);
   launch_k(k_prefill_attn<T, DH, DV>, grid, 128, smem, st, (const T*)q, (const T*)k, (const T*)v, (const T*)kpre,
-                                                      (const T*)vpre, npre, seq_off, tile_seq, tile_q0, pos0, Hq, Hkv,
-                                                      scale_log2, window, (T*)out);
+           (const T*)vpre, npre, seq_off, tile_seq, tile_q0, pos0, Hq, Hkv, scale_log2, window, (T*)out, ck);
   SR_LAUNCH();
   return SR_OK;
 }
@@ -997,9 +1032,10 @@ sr_status launch_decode_attention(int et, const void* q, const void* pool_layer,
 
 sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* kpre,
                                        const float* vpre, int npre, const int* seq_off, int n_seq, int rows, int pos0,
-                                       int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st) {
+                                       int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st,
+                                       CachedKeys ck, int max_cached) {
   if (rows == 0) return SR_OK;
-  const int max_keys = npre + rows;
+  const int max_keys = npre + max_cached + rows;
   const size_t smem = (size_t)max_keys * sizeof(float);
   if (smem > 200 * 1024) return set_err(SR_ERR_UNSUPPORTED, "fp32 prefill attention: %d keys too many", max_keys);
   static size_t attr = 48 * 1024;
@@ -1008,7 +1044,7 @@ sr_status launch_prefill_attention_f32(const float* q, const float* k, const flo
     attr = smem;
   }
   launch_k(k_prefill_attn_f32, dim3(rows, Hq), 128, smem, st, q, k, v, kpre, vpre, npre, seq_off, n_seq, pos0, Hq, Hkv, dh,
-                                                        1.f / sqrtf((float)dh), window, out);
+           1.f / sqrtf((float)dh), window, out, ck);
   SR_LAUNCH();
   return SR_OK;
 }
@@ -1016,7 +1052,7 @@ sr_status launch_prefill_attention_f32(const float* q, const float* k, const flo
 sr_status launch_prefill_attention(int et, const void* q, const void* k, const void* v, const void* kpre,
                                    const void* vpre, int npre, const int* seq_off, int n_seq, const int* tile_seq,
                                    const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
-                                   void* out, cudaStream_t st) {
+                                   void* out, cudaStream_t st, CachedKeys ck) {
   (void)n_seq;
   if (n_tiles == 0) return SR_OK;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "prefill attention: n_heads %% n_kv_heads != 0");
@@ -1024,13 +1060,13 @@ sr_status launch_prefill_attention(int et, const void* q, const void* k, const v
 #define SR_PRE(T)                                                                                                      \
   switch (dh) {                                                                                                        \
     case 32: return prefill_t<T, 32, 32>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, \
-                                         window, out, st);                                                            \
+                                         window, out, st, ck);                                                            \
     case 64: return prefill_t<T, 64, 64>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, \
-                                         window, out, st);                                                            \
+                                         window, out, st, ck);                                                            \
     case 128: return prefill_t<T, 128, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, \
-                                            Hkv, window, out, st);                                                    \
+                                            Hkv, window, out, st, ck);                                                    \
     case 256: return prefill_t<T, 256, 128>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, \
-                                            Hkv, window, out, st);                                                    \
+                                            Hkv, window, out, st, ck);                                                    \
   }
   if (et == SR_DT_F16) {
     SR_PRE(f16)

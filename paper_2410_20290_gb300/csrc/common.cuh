@@ -175,7 +175,9 @@ struct KvSink {        // where a layer's new K/V rows go besides the contiguous
   void* pool_layer;    // this layer's page 0 in the pool, or nullptr
   const int* page_table;
   int pt_stride;
-  const int* row_seq;  // page-table row per input row (nullptr: row 0 for every input row)
+  const int* row_seq;  // page-table row per input row (nullptr: row 0 for every input row; < 0: not stored)
+  int pos_base = 0;    // the pool pages hold positions pos_base, pos_base + 1, ... (page index (pos - pos_base) / 16)
+  const int* n_rows = nullptr;  // device count: rows >= *n_rows write nothing to the pool (nullptr: every row)
 };
 sr_status launch_rope_store(int dtype, const float* qkv, int M, const int* positions, const float2* rope, int Hq,
                             int Hkv, int dh, void* q_out, void* k_out, void* v_out, KvSink sink, cudaStream_t st);
@@ -189,7 +191,8 @@ sr_status launch_copy_page(int dtype, void* pool, long long layer_stride_elems, 
 sr_status launch_sample(const float* logits, long long ld, int b, int V, const int* orig_ids, const int* steps,
                         uint64_t seed, float temperature, float eos_bias, int eos_id, int* tokens_out,
                         int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st,
-                        double* lp_sum = nullptr);  // lp_sum: += ln p(token) per candidate id (Section 5.3 reward)
+                        double* lp_sum = nullptr,   // lp_sum: += ln p(token) per candidate id (Section 5.3 reward)
+                        const int* n_rows = nullptr);  // device count: rows >= *n_rows are skipped
 
 // attention.cu
 // shared_pos > 0: positions [0, shared_pos) sit in pages shared by every row's page table (the prompt);
@@ -203,13 +206,25 @@ sr_status launch_decode_attention(int dtype, const void* q, const void* pool_lay
 int decode_attention_max_splits(int max_len);
 int decode_attention_slots(int max_len, int window, int shared_pos);
 size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits);
+// Keys of a prefill sequence that sit between the shared prefix and the sequence's own rows: positions
+// pos0 .. pos0 + seq_cached[j] - 1 of sequence j, kept in a paged pool ([page][2 (K, V)][Hkv][16][dh] per
+// layer) under page-table row seq_cand[j]; the sequence's own rows then start at position pos0 + seq_cached[j].
+// pool == nullptr: no such keys.
+struct CachedKeys {
+  const void* pool = nullptr;  // this layer's page 0
+  const int* page_table = nullptr;
+  int pt_stride = 0;
+  const int* seq_cand = nullptr;
+  const int* seq_cached = nullptr;
+};
 sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* k_pre,
                                        const float* v_pre, int n_pre, const int* seq_off, int n_seq, int rows,
-                                       int pos0, int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st);
+                                       int pos0, int Hq, int Hkv, int dh, int window, float* out, cudaStream_t st,
+                                       CachedKeys ck = CachedKeys(), int max_cached = 0);  // max_cached >= seq_cached[]
 sr_status launch_prefill_attention(int et, const void* q, const void* k, const void* v, const void* k_pre,
                                    const void* v_pre, int n_pre, const int* seq_off, int n_seq, const int* tile_seq,
                                    const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
-                                   void* out, cudaStream_t st);
+                                   void* out, cudaStream_t st, CachedKeys ck = CachedKeys());
 // elementwise.cu: in-place bf16 -> fp16 conversion of n elements (weights at load)
 sr_status launch_bf16_to_f16(void* p, size_t n, cudaStream_t st);
 

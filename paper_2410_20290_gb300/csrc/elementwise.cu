@@ -145,12 +145,15 @@ __global__ void k_rope_store(const float* __restrict__ qkv, const int* __restric
   const float* row = qkv + (size_t)r * W;
   T* pk = nullptr;
   T* pv = nullptr;
-  if (sink.pool_layer) {
+  if (sink.pool_layer && (!sink.n_rows || r < *sink.n_rows)) {
     const int seq = sink.row_seq ? sink.row_seq[r] : 0;
-    const int page = sink.page_table[(size_t)seq * sink.pt_stride + pos / PAGE];
-    T* base = reinterpret_cast<T*>(sink.pool_layer) + (size_t)page * 2 * Hkv * PAGE * dh + (size_t)(pos % PAGE) * dh;
-    pk = base;
-    pv = base + (size_t)Hkv * PAGE * dh;
+    if (seq >= 0) {
+      const int pp = pos - sink.pos_base;
+      const int page = sink.page_table[(size_t)seq * sink.pt_stride + pp / PAGE];
+      T* base = reinterpret_cast<T*>(sink.pool_layer) + (size_t)page * 2 * Hkv * PAGE * dh + (size_t)(pp % PAGE) * dh;
+      pk = base;
+      pv = base + (size_t)Hkv * PAGE * dh;
+    }
   }
   // rotated heads: Hq query heads then Hkv key heads, pairs (i, i + half)
   for (int idx = threadIdx.x; idx < (Hq + Hkv) * half; idx += blockDim.x) {
@@ -203,12 +206,15 @@ __global__ void __launch_bounds__(256) k_rope_store_v(const float* __restrict__ 
   const float* row = qkv + (size_t)r * (Hq + 2 * Hkv) * dh;
   T* pk = nullptr;
   T* pv = nullptr;
-  if (sink.pool_layer) {
+  if (sink.pool_layer && (!sink.n_rows || r < *sink.n_rows)) {
     const int seq = sink.row_seq ? sink.row_seq[r] : 0;
-    const int page = sink.page_table[(size_t)seq * sink.pt_stride + pos / PAGE];
-    T* base = reinterpret_cast<T*>(sink.pool_layer) + (size_t)page * 2 * Hkv * PAGE * dh + (size_t)(pos % PAGE) * dh;
-    pk = base;
-    pv = base + (size_t)Hkv * PAGE * dh;
+    if (seq >= 0) {
+      const int pp = pos - sink.pos_base;
+      const int page = sink.page_table[(size_t)seq * sink.pt_stride + pp / PAGE];
+      T* base = reinterpret_cast<T*>(sink.pool_layer) + (size_t)page * 2 * Hkv * PAGE * dh + (size_t)(pp % PAGE) * dh;
+      pk = base;
+      pv = base + (size_t)Hkv * PAGE * dh;
+    }
   }
   for (int idx = threadIdx.x; idx < (Hq + Hkv) * gph; idx += blockDim.x) {
     const int h = idx / gph, i = (idx % gph) * 4;

@@ -328,6 +328,14 @@ struct PrefillPlan {
   const char* pre_k = nullptr;    // per-layer prefix K / V stores: base + l * layer_stride
   const char* pre_v = nullptr;
   size_t pre_layer_bytes = 0;
+  // cached keys between the prefix and each sequence's own rows (reward-model KV kept across rounds)
+  const char* cache_pool = nullptr;  // layer 0 page 0; layer l at + l * cache_layer_bytes
+  size_t cache_layer_bytes = 0;
+  const int* cache_pt = nullptr;
+  int cache_pt_stride = 0;
+  const int* seq_cand = nullptr;     // device [n_seq]
+  const int* seq_cached = nullptr;   // device [n_seq]
+  int max_cached = 0;
 };
 // Where a prefill's per-layer K/V goes.
 struct PrefillKv {
@@ -336,7 +344,10 @@ struct PrefillKv {
   size_t store_layer_bytes = 0;
   void* pool = nullptr;           // paged pool (layer 0 page 0) or nullptr
   size_t pool_layer_bytes = 0;
-  const int* page_row = nullptr;  // page table row for positions (row_seq = null)
+  const int* page_row = nullptr;  // page table: one row for every input row (row_seq = null) ...
+  int pt_stride = 0;
+  const int* row_seq = nullptr;   // ... or row row_seq[r] for input row r (< 0: not stored)
+  int pos_base = 0;               // positions held by the pages start here
 };
 
 sr_status linear(const Model& m, const void* A, const void* W, void* C, int M, int N, int K, int epi,
@@ -384,13 +395,23 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
     char* kout = kv.store_k ? kv.store_k + l * kv.store_layer_bytes : w.k;
     char* vout = kv.store_v ? kv.store_v + l * kv.store_layer_bytes : w.v;
     KvSink sink{nullptr, nullptr, 0, nullptr};
-    if (kv.pool) sink = KvSink{static_cast<char*>(kv.pool) + l * kv.pool_layer_bytes, kv.page_row, 0, nullptr};
+    if (kv.pool)
+      sink = KvSink{static_cast<char*>(kv.pool) + l * kv.pool_layer_bytes, kv.page_row, kv.pt_stride, kv.row_seq,
+                    kv.pos_base};
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
       SR_TRY(launch_rope_store(m.et, w.qkv, M, pos, m.rope, Hq, Hkv, dh, w.q, kout, vout, sink, st));
     }
     const char* pk = plan.n_pre ? plan.pre_k + l * plan.pre_layer_bytes : nullptr;
     const char* pv = plan.n_pre ? plan.pre_v + l * plan.pre_layer_bytes : nullptr;
+    CachedKeys ck;
+    if (plan.cache_pool) {
+      ck.pool = plan.cache_pool + l * plan.cache_layer_bytes;
+      ck.page_table = plan.cache_pt;
+      ck.pt_stride = plan.cache_pt_stride;
+      ck.seq_cand = plan.seq_cand;
+      ck.seq_cached = plan.seq_cached;
+    }
     const double kvb = (double)m.kv_tok_elems() * m.esz;
     {
       Scope sa(pf, SR_KC_ATTN_PREFILL, st, attn_flops,
@@ -398,11 +419,12 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
       if (m.et == SR_DT_F16)
         SR_TRY(launch_prefill_attention(m.et, w.q, kout, vout, pk, pv, plan.n_pre, plan.seq_off, plan.n_seq,
                                         plan.tile_seq, plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window,
-                                        w.att, st));
+                                        w.att, st, ck));
       else
         SR_TRY(launch_prefill_attention_f32((const float*)w.q, (const float*)kout, (const float*)vout,
                                             (const float*)pk, (const float*)pv, plan.n_pre, plan.seq_off, plan.n_seq,
-                                            M, plan.pos0, Hq, Hkv, dh, d.window, (float*)w.att, st));
+                                            M, plan.pos0, Hq, Hkv, dh, d.window, (float*)w.att, st, ck,
+                                            plan.max_cached));
     }
     SR_TRY(linear(m, w.att, lw.wo, w.x, M, D, Hq * dh, EPI_ADD_F32, st, pf, gcls));
     {
@@ -414,12 +436,15 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
   return SR_OK;
 }
 
-// algorithmic flops of causal prefill attention: query i of a sequence sees n_pre + i + 1 keys
-double prefill_attn_flops(const Model& m, const std::vector<int>& taus, size_t s0, size_t n, int n_pre) {
+// algorithmic flops of causal prefill attention: new row i of a sequence with c cached positions sees
+// n_pre + c + i + 1 keys (c = 0 without a cache)
+double prefill_attn_flops(const Model& m, const std::vector<int>& taus, size_t s0, size_t n, int n_pre,
+                          const std::vector<int>* cached = nullptr) {
   double keys = 0;
   for (size_t j = s0; j < s0 + n; ++j) {
-    const double t = taus[j];
-    keys += t * n_pre + t * (t + 1) / 2;
+    const double c = cached ? (*cached)[j] : 0;
+    const double t = taus[j] - c;  // new rows
+    keys += t * (n_pre + c) + t * (t + 1) / 2;
   }
   return 4.0 * m.d.n_heads * m.d.head_dim * keys;  // per layer
 }
@@ -444,6 +469,16 @@ struct sr_ctx {
   // reward-model prompt KV store [layer][P][Hkv][dh] (K and V)
   char *rm_pk = nullptr, *rm_pv = nullptr;
   size_t c_rm_pk = 0, c_rm_pv = 0;
+  // reward-model KV of response positions kept across rounds: [layer][page][2][Hkv][16][dh], page table
+  // rm_pt [N][rm_max_pages] (device; host mirror and free stack in the batch)
+  size_t rm_cache_bytes_req = 0;
+  char* rm_pool = nullptr;
+  int rm_pool_cap = 0;          // pages allocated
+  size_t rm_page_bytes = 0;
+  int* rm_pt = nullptr;
+  size_t c_rm_pt = 0;
+  int* row_cand = nullptr;      // scoring rows -> candidate whose cache receives the row (-1: not stored)
+  size_t c_row_cand = 0;
   // candidate state
   size_t c_len = 0, c_status = 0, c_tok = 0, c_pt = 0, c_live = 0, c_rset = 0, c_free = 0, c_tokin = 0, c_posin = 0,
          c_kvlen = 0, c_tail = 0, c_prow = 0, c_ids = 0, c_reward = 0, c_rr = 0, c_logits = 0, c_mask = 0, c_prompt = 0,
@@ -468,6 +503,18 @@ struct sr_ctx {
   sr::Prof prof;
 };
 
+// Host bookkeeping of the reward-model KV cache of one batch: which response positions of each
+// candidate have their reward-model K/V in the cache pool, and the pages that hold them.
+struct RmCache {
+  bool on = false;
+  int pages = 0, max_pages = 0;     // pool pages; pages per candidate (ceil(max_new / 16))
+  std::vector<int> free_stack;      // LIFO, top at the back
+  std::vector<int> cached;          // [N] positions 0 .. cached - 1 are in the cache
+  std::vector<int> held;            // [N] pages held
+  std::vector<int> pt;              // [N][max_pages] host mirror of the device page table
+  long long reused = 0;             // positions read from the cache instead of recomputed
+};
+
 struct sr_batch {
   int P = 0, N = 0, max_new = 0, eos_id = -1, n_sh = 0, has_tail = 0, max_pages = 0, n_pages = 0;
   float temperature = 1.f, eos_bias = 0.f;
@@ -475,6 +522,7 @@ struct sr_batch {
   int n_live = 0, n_rset = 0, g = 0;  // g: tokens generated by every live candidate
   bool active = false;
   int reward_kind = SR_REWARD_MODEL;  // the context's reward kind when the batch started
+  RmCache rmc;
 };
 
 namespace sr {
@@ -661,7 +709,10 @@ sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
 }
 
 // One batched decode step of every live candidate (positions P + g - 1), Eq. auto-regressive.
-sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
+// sync = false enqueues the step without reading the control words back: the launches are sized for
+// b.n_live, an upper bound of the live count (candidates only complete between rounds), and the kernels
+// that write candidate state skip the slots past the device's live count.
+sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host, bool sync = true) {
   const Model& m = c->gen;
   const sr_model_desc& d = m.d;
   Work& w = c->wg;
@@ -703,7 +754,7 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
     {
       Scope sc(pf, SR_KC_ELEMENTWISE, st);
       SR_TRY(launch_rope_store(m.et, w.qkv, n, c->pos_in, m.rope, Hq, Hkv, dh, w.q, nullptr, nullptr,
-                               KvSink{pool_l, c->pt, b.max_pages, c->live}, st));
+                               KvSink{pool_l, c->pt, b.max_pages, c->live, 0, c->ctrl + C_NLIVE}, st));
     }
     {
       Scope sc(pf, SR_KC_ATTN_DECODE, st, attn_flops, attn_bytes);
@@ -729,26 +780,34 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host) {
     Scope sc(pf, SR_KC_SAMPLE, st, 0, 4.0 * n * d.vocab);
     SR_TRY(launch_sample(c->logits, d.vocab, n, d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias,
                          b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, st,
-                         b.reward_kind == SR_REWARD_LOGPROB ? c->lp_sum : nullptr));
+                         b.reward_kind == SR_REWARD_LOGPROB ? c->lp_sum : nullptr, c->ctrl + C_NLIVE));
   }
   {
     Scope sc(pf, SR_KC_CONTROL, st);
     SR_TRY(ctl_step_end(b.P, b.n_sh, c->live, c->ctrl, c->len, c->status, c->pt, b.max_pages, c->free_stack, st));
   }
+  b.g += 1;
+  if (!sync) return SR_OK;
   SR_TRY(read_ctrl(c));
   b.n_live = c->h_ctrl[C_NLIVE];
-  b.g += 1;
   return SR_OK;
 }
 
-__global__ void k_gather_rows(const int* __restrict__ ids, const int* __restrict__ off, const int* __restrict__ tok,
-                              int max_new, int P, int* tok_rows, int* pos_rows, int* last_row) {
+// Reward-model input rows of one scoring chunk: sequence j (candidate ids[j]) contributes its response
+// tokens cached[j] .. cached[j] + n - 1 at positions P + cached[j] + i; row_cand receives the candidate id
+// where the rows' K/V go to the cache (store[j] != 0), else -1.
+__global__ void k_gather_rows(const int* __restrict__ ids, const int* __restrict__ off, const int* __restrict__ cached,
+                              const int* __restrict__ store, const int* __restrict__ tok, int max_new, int P,
+                              int* tok_rows, int* pos_rows, int* row_cand, int* last_row) {
   pdl_entry();
   const int j = blockIdx.x;
   const int id = ids[j], r0 = off[j], n = off[j + 1] - off[j];
+  const int c = cached ? cached[j] : 0;
+  const int rc = (row_cand && store[j]) ? id : -1;
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    tok_rows[r0 + i] = tok[(size_t)id * max_new + i];
-    pos_rows[r0 + i] = P + i;
+    tok_rows[r0 + i] = tok[(size_t)id * max_new + c + i];
+    pos_rows[r0 + i] = P + c + i;
+    if (row_cand) row_cand[r0 + i] = rc;
   }
   if (threadIdx.x == 0) last_row[j] = r0 + n - 1;
 }
@@ -764,11 +823,26 @@ __global__ void k_mean_logprob(const int* __restrict__ ids_taus, int n, const do
 
 constexpr int CHUNK_ROWS = 16384;  // reward-model rows (response tokens) per scoring pass
 
+// Give back the cache pages of every candidate that may not keep them (not in `keep`), in ascending
+// (candidate id, page index) order.
+void rm_cache_release(RmCache& rc, const std::vector<char>& keep) {
+  for (size_t id = 0; id < rc.held.size(); ++id) {
+    if (keep[id] || rc.held[id] == 0) continue;
+    for (int p = 0; p < rc.held[id]; ++p) rc.free_stack.push_back(rc.pt[id * rc.max_pages + p]);
+    rc.held[id] = 0;
+    rc.cached[id] = 0;
+  }
+}
+
 // Rewards s(X ++ Y_k^{<= tau_k}) for candidates ids_h[0..n) with tau_k = taus[k] (Eq.
 // partial.reward.set); results into rewards_dev[0..n).  Each chunk runs the reward model over the
-// packed response tokens, attending to the prompt KV computed once at prefill.
+// packed response tokens, attending to the prompt KV computed once at prefill.  With the reward-model
+// cache on, positions already in the cache are not run again: a candidate's new rows start at its cached
+// length (one row at least) and attend to the prompt, its cached pages and each other; when `store` is
+// set (a rejection round), the new rows' K/V are added to the cache for every candidate the free pages
+// can serve, in ascending id order, so that a later round or the final scoring reads them.
 sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std::vector<int>& taus,
-                float* rewards_dev) {
+                float* rewards_dev, bool store, long long* rm_rows = nullptr) {
   const Model& r = c->rm;
   const int n = (int)ids_h.size();
   if (n == 0) return SR_OK;
@@ -785,7 +859,40 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
     return SR_OK;
   }
   const size_t rm_layer = (size_t)b.P * r.kv_tok_elems() * r.esz;
-  // plan chunks on the host: [ids | off | tiles_seq | tiles_q0] per chunk in one pinned buffer
+  RmCache& rc = b.rmc;
+  SR_CUDA(cudaStreamSynchronize(c->st));  // host staging and the page-table mirror may feed earlier copies
+  // new rows per candidate, and where their K/V go
+  std::vector<int> cached(n, 0), newr(n), st_flag(n, 0);
+  if (rc.on) {
+    std::vector<char> keep(rc.held.size(), 0);
+    for (int id : ids_h) keep[id] = 1;
+    rm_cache_release(rc, keep);
+    for (int j = 0; j < n; ++j) cached[j] = std::min(rc.cached[ids_h[j]], taus[j] - 1);
+    if (store) {
+      for (int j = 0; j < n; ++j) {
+        const int id = ids_h[j];
+        const int need = std::max(0, (taus[j] + PAGE - 1) / PAGE - rc.held[id]);
+        if (need > (int)rc.free_stack.size()) continue;
+        for (int p = 0; p < need; ++p) {
+          rc.pt[(size_t)id * rc.max_pages + rc.held[id] + p] = rc.free_stack.back();
+          rc.free_stack.pop_back();
+        }
+        rc.held[id] += need;
+        st_flag[j] = 1;
+      }
+      SR_CUDA(cudaMemcpyAsync(c->rm_pt, rc.pt.data(), rc.pt.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+    }
+  }
+  long long rows_total = 0;
+  int max_cached = 0;
+  for (int j = 0; j < n; ++j) {
+    newr[j] = taus[j] - cached[j];
+    rows_total += newr[j];
+    rc.reused += cached[j];
+    max_cached = std::max(max_cached, cached[j]);
+  }
+  if (rm_rows) *rm_rows += rows_total;
+  // plan chunks on the host: [ids | off | cached | store | tiles_seq | tiles_q0] per chunk in one pinned buffer
   struct Chunk {
     int s0, ns, rows, n_tiles;
     size_t meta;
@@ -794,16 +901,15 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
   size_t meta_len = 0;
   for (int s = 0; s < n;) {
     Chunk ch{s, 0, 0, 0, meta_len};
-    while (s < n && (ch.ns == 0 || ch.rows + taus[s] <= CHUNK_ROWS)) {
-      ch.rows += taus[s];
-      ch.n_tiles += (taus[s] + 63) / 64;
+    while (s < n && (ch.ns == 0 || ch.rows + newr[s] <= CHUNK_ROWS)) {
+      ch.rows += newr[s];
+      ch.n_tiles += (newr[s] + 63) / 64;
       ++ch.ns;
       ++s;
     }
-    meta_len += (size_t)ch.ns + (ch.ns + 1) + 2 * (size_t)ch.n_tiles;
+    meta_len += 3 * (size_t)ch.ns + (ch.ns + 1) + 2 * (size_t)ch.n_tiles;
     chunks.push_back(ch);
   }
-  SR_CUDA(cudaStreamSynchronize(c->st));
   SR_TRY(grow_host(c->h_meta, c->c_hmeta, meta_len));
   SR_TRY(grow(c->meta, c->c_meta, meta_len));
   int max_rows = 0;
@@ -811,34 +917,43 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
     int* h = c->h_meta + ch.meta;
     int* hid = h;
     int* hoff = h + ch.ns;
-    int* hts = hoff + ch.ns + 1;
+    int* hc = hoff + ch.ns + 1;
+    int* hst = hc + ch.ns;
+    int* hts = hst + ch.ns;
     int* htq = hts + ch.n_tiles;
     int o = 0, t = 0;
     for (int j = 0; j < ch.ns; ++j) {
       hid[j] = ids_h[ch.s0 + j];
       hoff[j] = o;
-      const int tau = taus[ch.s0 + j];
-      for (int q0 = 0; q0 < tau; q0 += 64) hts[t] = j, htq[t] = q0, ++t;
-      o += tau;
+      hc[j] = cached[ch.s0 + j];
+      hst[j] = st_flag[ch.s0 + j];
+      const int nr = newr[ch.s0 + j];
+      for (int q0 = 0; q0 < nr; q0 += 64) hts[t] = j, htq[t] = q0, ++t;
+      o += nr;
     }
     hoff[ch.ns] = o;
     max_rows = std::max(max_rows, ch.rows);
   }
   SR_CUDA(cudaMemcpyAsync(c->meta, c->h_meta, meta_len * sizeof(int), cudaMemcpyHostToDevice, c->st));
   SR_TRY(c->wr.ensure(r, max_rows));
+  if (rc.on) SR_TRY(grow(c->row_cand, c->c_row_cand, (size_t)max_rows));
   // token / position rows for the largest chunk
   int *tok_rows = nullptr, *pos_rows = nullptr;
   SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&tok_rows), (size_t)max_rows * sizeof(int), c->st));
   SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&pos_rows), (size_t)max_rows * sizeof(int), c->st));
+  const size_t cache_layer = (size_t)rc.pages * c->rm_page_bytes;
   sr_status status = SR_OK;
   for (const Chunk& ch : chunks) {
     const int* did = c->meta + ch.meta;
     const int* doff = did + ch.ns;
-    const int* dts = doff + ch.ns + 1;
+    const int* dc = doff + ch.ns + 1;
+    const int* dst = dc + ch.ns;
+    const int* dts = dst + ch.ns;
     const int* dtq = dts + ch.n_tiles;
     {
       Scope sc(&c->prof, SR_KC_ELEMENTWISE, c->st);
-      launch_k(k_gather_rows, ch.ns, 128, 0, c->st, did, doff, c->tok, b.max_new, b.P, tok_rows, pos_rows, c->last_row);
+      launch_k(k_gather_rows, ch.ns, 128, 0, c->st, did, doff, rc.on ? dc : (const int*)nullptr, dst, c->tok,
+               b.max_new, b.P, tok_rows, pos_rows, rc.on ? c->row_cand : (int*)nullptr, c->last_row);
     }
     if ((status = [&]() -> sr_status { SR_LAUNCH(); return SR_OK; }()) != SR_OK) break;
     PrefillPlan plan;
@@ -852,8 +967,26 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
     plan.pre_k = c->rm_pk;
     plan.pre_v = c->rm_pv;
     plan.pre_layer_bytes = rm_layer;
-    if ((status = forward_prefill(r, c->wr, ch.rows, tok_rows, pos_rows, plan, PrefillKv(), c->st, &c->prof,
-                                  SR_KC_GEMM_SCORE, prefill_attn_flops(r, taus, ch.s0, ch.ns, b.P))) != SR_OK)
+    PrefillKv kv;
+    if (rc.on) {
+      plan.cache_pool = c->rm_pool;
+      plan.cache_layer_bytes = cache_layer;
+      plan.cache_pt = c->rm_pt;
+      plan.cache_pt_stride = rc.max_pages;
+      plan.seq_cand = did;
+      plan.seq_cached = dc;
+      plan.max_cached = max_cached;
+      if (store) {
+        kv.pool = c->rm_pool;
+        kv.pool_layer_bytes = cache_layer;
+        kv.page_row = c->rm_pt;
+        kv.pt_stride = rc.max_pages;
+        kv.row_seq = c->row_cand;
+        kv.pos_base = b.P;
+      }
+    }
+    if ((status = forward_prefill(r, c->wr, ch.rows, tok_rows, pos_rows, plan, kv, c->st, &c->prof, SR_KC_GEMM_SCORE,
+                                  prefill_attn_flops(r, taus, ch.s0, ch.ns, b.P, &cached))) != SR_OK)
       break;
     Scope sc(&c->prof, SR_KC_ELEMENTWISE, c->st);
     if ((status = launch_score_head(r.et, r.d.norm, c->wr.x, c->last_row, ch.ns, r.final_w, r.final_b,
@@ -862,6 +995,9 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
   }
   cudaFreeAsync(tok_rows, c->st);
   cudaFreeAsync(pos_rows, c->st);
+  if (status == SR_OK && rc.on && store)
+    for (int j = 0; j < n; ++j)
+      if (st_flag[j]) rc.cached[ids_h[j]] = taus[j];
   return status;
 }
 
@@ -893,6 +1029,37 @@ sr_status validate_common(const sr_ctx* c, int P, int N, int max_new, float temp
   return SR_OK;
 }
 
+// The reward-model KV cache of this batch (off unless sr_set_rm_cache gave it bytes and the reward model
+// scores): pages = floor(bytes / (16 positions x the reward model's KV bytes per position)).
+sr_status prepare_rm_cache(sr_ctx* c, sr_batch& b) {
+  RmCache& rc = b.rmc;
+  rc = RmCache();
+  if (c->rm_cache_bytes_req == 0 || b.reward_kind != SR_REWARD_MODEL) return SR_OK;
+  const Model& r = c->rm;
+  c->rm_page_bytes = (size_t)2 * r.d.n_kv_heads * PAGE * r.d.head_dim * r.esz;
+  const size_t per_page = c->rm_page_bytes * r.d.n_layers;
+  const long long pages = (long long)(c->rm_cache_bytes_req / per_page);
+  if (pages < 1) return SR_OK;  // too small for one page: no cache
+  if (pages > (1ll << 30)) return set_err(SR_ERR_INVALID_ARG, "reward-model cache too large");
+  if (c->rm_pool_cap != (int)pages) {
+    if (c->rm_pool) cudaFree(c->rm_pool);
+    c->rm_pool = nullptr;
+    c->rm_pool_cap = 0;
+    SR_CUDA(cudaMalloc(&c->rm_pool, (size_t)pages * per_page));
+    c->rm_pool_cap = (int)pages;
+  }
+  rc.on = true;
+  rc.pages = (int)pages;
+  rc.max_pages = (b.max_new + PAGE - 1) / PAGE;
+  rc.free_stack.resize(rc.pages);
+  for (int i = 0; i < rc.pages; ++i) rc.free_stack[i] = i;  // LIFO: the first page taken is the highest
+  rc.cached.assign(b.N, 0);
+  rc.held.assign(b.N, 0);
+  rc.pt.assign((size_t)b.N * rc.max_pages, 0);
+  SR_TRY(grow(c->rm_pt, c->c_rm_pt, rc.pt.size()));
+  return SR_OK;
+}
+
 sr_status begin(sr_ctx* c, sr_batch& b, const int32_t* prompt, bool prompt_on_device, int P, int N, int max_new,
                 float temperature, float eos_bias, int eos_id, uint64_t seed) {
   SR_TRY(validate_common(c, P, N, max_new, temperature, eos_id));
@@ -906,6 +1073,7 @@ sr_status begin(sr_ctx* c, sr_batch& b, const int32_t* prompt, bool prompt_on_de
   b.max_pages = (P + max_new - 1) / PAGE + 1;
   SR_TRY(prepare_pool(c, b));
   SR_TRY(prepare_state(c, b));
+  SR_TRY(prepare_rm_cache(c, b));
   SR_TRY(grow(c->prompt, c->c_prompt, (size_t)P));
   SR_CUDA(cudaMemcpyAsync(c->prompt, prompt, P * sizeof(int), prompt_on_device ? cudaMemcpyDeviceToDevice
                                                                               : cudaMemcpyHostToDevice, c->st));
@@ -955,11 +1123,10 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
         if (trig) {
           double ts = now_ms();
           SR_TRY(read_rset(c, b, ids, taus, nullptr));
-          SR_TRY(score(c, b, ids, taus, c->rr));
+          SR_TRY(score(c, b, ids, taus, c->rr, true, &S.rm_tokens));
           SR_CUDA(cudaStreamSynchronize(c->st));
           double tsel = now_ms();
           S.ms_score += tsel - ts;
-          for (int t : taus) S.rm_tokens += t;
           {
             Scope sc(&c->prof, SR_KC_CONTROL, c->st);
             SR_TRY(ctl_round(b.P, b.n_sh, alpha, pool_mode && need ? 1 : 0, c->rr, c->rset, c->live, c->ctrl,
@@ -983,8 +1150,12 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
         }
       }
       if (need && c->h_ctrl[C_TOP] < b.n_live) return set_err(SR_ERR_OOM, "KV pool cannot hold the next decode step");
+      // Between page boundaries no memory trigger can fire and no step needs a page, so the next steps are
+      // enqueued without reading the live count back; the host syncs before a step that opens a page and
+      // when the candidates reach max_new.
+      const bool sync = (b.P + b.g) % PAGE == 0 || b.g + 1 >= b.max_new;
       double td = now_ms();
-      SR_TRY(decode_step(c, b, nullptr));
+      SR_TRY(decode_step(c, b, nullptr, sync));
       S.ms_decode += now_ms() - td;
       S.decode_steps++;
     }
@@ -995,16 +1166,16 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
     for (size_t i = 0; i < ids.size(); ++i)
       if (stat[i] == ST_PENDING) pid.push_back(ids[i]), ptau.push_back(taus[i]);
     if (!pid.empty()) {
-      SR_TRY(score(c, b, pid, ptau, c->rr));
+      SR_TRY(score(c, b, pid, ptau, c->rr, false, &S.rm_tokens));
       SR_CUDA(cudaMemcpyAsync(c->ids, pid.data(), pid.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
       SR_TRY(ctl_mark_done(c->ids, c->rr, (int)pid.size(), c->status, c->reward, c->st));
       SR_CUDA(cudaStreamSynchronize(c->st));
-      for (int t : ptau) S.rm_tokens += t;
     }
     S.ms_score += now_ms() - tf;
   }
   S.rm_tokens += b.P;
   if (b.reward_kind != SR_REWARD_MODEL) S.rm_tokens = 0;  // the generator scored itself
+  S.rm_tokens_cached = b.rmc.reused;
   SR_TRY(ctl_final(b.N, c->status, c->reward, c->tok, b.max_new, c->len, c->out_tok, c->d_outlen, c->ctrlf + 1,
                    c->ctrl, c->st));
   SR_TRY(read_ctrl(c));
@@ -1096,7 +1267,7 @@ void sr_destroy(sr_ctx* c) {
   free_model(c->rm);
   c->wg.release();
   c->wr.release();
-  void* dev[] = {c->pool, c->rm_pk, c->rm_pv, c->len, c->status, c->tok, c->pt, c->live, c->rset, c->free_stack,
+  void* dev[] = {c->pool, c->rm_pk, c->rm_pv, c->rm_pool, c->rm_pt, c->row_cand, c->len, c->status, c->tok, c->pt, c->live, c->rset, c->free_stack,
                  c->tok_in, c->pos_in, c->kv_len, c->tail_dst, c->prompt_row, c->ids, c->prompt, c->iota, c->meta,
                  c->out_tok, c->last_row, c->reward, c->rr, c->logits, c->logits0, c->mask, c->ctrl, c->ctrlf, c->d_score,
                  c->d_outlen};
@@ -1122,6 +1293,19 @@ sr_status sr_auto_b_init(const sr_model_desc* gen, size_t kv_pool_bytes, int P, 
   long long n = avail < 0 ? 0 : (per == 0 ? n_max : std::min<long long>(n_max, avail / per));
   *n_out = (int)n;
   if (n < 1) return set_err(SR_ERR_OOM, "sr_auto_b_init: the pool cannot hold one candidate to tau_min tokens");
+  return SR_OK;
+}
+
+sr_status sr_set_rm_cache(sr_ctx* c, size_t bytes) {
+  if (!c) return set_err(SR_ERR_INVALID_ARG, "null context");
+  c->rm_cache_bytes_req = bytes;
+  if (bytes == 0 && c->rm_pool) {
+    SR_CUDA(cudaSetDevice(c->device));
+    SR_CUDA(cudaStreamSynchronize(c->st));
+    cudaFree(c->rm_pool);
+    c->rm_pool = nullptr;
+    c->rm_pool_cap = 0;
+  }
   return SR_OK;
 }
 
@@ -1235,7 +1419,7 @@ sr_status sr_score_partial(sr_ctx* c, sr_batch* b, float* rewards, int* b_out) {
   if (!b->active) return set_err(SR_ERR_STATE, "batch not active");
   std::vector<int> ids, taus;
   SR_TRY(read_rset(c, *b, ids, taus, nullptr));
-  SR_TRY(score(c, *b, ids, taus, c->rr));
+  SR_TRY(score(c, *b, ids, taus, c->rr, true));
   SR_CUDA(cudaMemcpyAsync(rewards, c->rr, ids.size() * sizeof(float), cudaMemcpyDeviceToHost, c->st));
   SR_CUDA(cudaStreamSynchronize(c->st));
   if (b_out) *b_out = (int)ids.size();

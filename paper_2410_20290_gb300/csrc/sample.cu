@@ -71,8 +71,10 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
                                                     const int* __restrict__ orig_ids, const int* __restrict__ steps,
                                                     uint32_t k0, uint32_t k1, float temperature, float eos_bias,
                                                     int eos_id, int* __restrict__ tokens_out, int* tok_hist,
-                                                    int max_new, int* lens, int* status, double* lp_sum) {
+                                                    int max_new, int* lens, int* status, double* lp_sum,
+                                                    const int* __restrict__ n_rows) {
   pdl_entry();
+  if (n_rows && (int)blockIdx.x >= *n_rows) return;  // a slot past the live count the step started with
   __shared__ float s_best[THREADS / 32];
   __shared__ int s_idx[THREADS / 32];
   __shared__ float s_m[THREADS / 32], s_s[THREADS / 32];
@@ -165,12 +167,12 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
 
 sr_status launch_sample(const float* logits, long long ld, int b, int V, const int* orig_ids, const int* steps,
                         uint64_t seed, float temperature, float eos_bias, int eos_id, int* tokens_out, int* tok_hist,
-                        int max_new, int* lens, int* status, cudaStream_t st, double* lp_sum) {
+                        int max_new, int* lens, int* status, cudaStream_t st, double* lp_sum, const int* n_rows) {
   if (b == 0) return SR_OK;
   if (!(temperature > 0.f)) return set_err(SR_ERR_INVALID_ARG, "temperature must be > 0");
   launch_k(k_sample, b, THREADS, 0, st, logits, ld, V, orig_ids, steps, (uint32_t)(seed & 0xFFFFFFFFu),
                                   (uint32_t)(seed >> 32), temperature, eos_bias, eos_id, tokens_out, tok_hist, max_new,
-                                  lens, status, lp_sum);
+                                  lens, status, lp_sum, n_rows);
   SR_LAUNCH();
   return SR_OK;
 }
