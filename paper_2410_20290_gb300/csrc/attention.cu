@@ -19,6 +19,7 @@
 #include <type_traits>
 
 #include "common.cuh"
+#include "tma.cuh"
 
 namespace sr {
 namespace {
@@ -467,6 +468,1005 @@ __global__ void __launch_bounds__(128) k_decode_attn_tc(const T* __restrict__ q,
   }
 }
 
+// ------------------------------------------------------------------------------------------------
+// Streaming paged decode attention (16-bit KV, head_dim 128, 8 kv heads, G query heads per kv head).
+//
+// All (row, page) work of one launch is laid out row by row (row s contributes the pages of its positions
+// [t_lo, L)) and cut into gridDim.x contiguous shares of (almost) equal page counts; one persistent CTA per
+// SM walks its share in order, so short and long rows alike keep every SM's copy stream full and no row
+// pays a launch or pipeline fill of its own.  Warp 8 (one lane) is the producer: per page it issues four
+// 128-byte-swizzled TMA copies (K and V of all 8 kv heads, each as two 64-column halves, 64 KB) into a
+// 3-stage ring.  Warps 0..7 are the consumers, warp h serving kv head h: S^T = K Q^T per page with
+// mma.sync (16 positions x 8 head columns: the G query heads, zero-padded), the online softmax over the
+// 8 lanes holding a head column, and O^T += V^T P^T, exactly as the per-row kernel does.  A row whose pages
+// lie inside the share is finalised by the CTA (folding in the shared-prefix partial when there is one).
+// A row cut by a share boundary leaves (O, m, l) partials, at most two per CTA (its first and last
+// segment); each consumer warp counts its finished segment on a per-(row, kv head) counter and the last
+// one merges the row's partials in a fixed order (prefix, then the CTAs in order), so the result does not
+// depend on which CTA finishes last, and resets the counter.  No CTA waits on another.
+constexpr int ST_HKV = 8, ST_DH = 128, ST_STAGES = 3;
+constexpr int ST_TILE = ST_HKV * PAGE * 64 * 2;  // one 64-column half of a page's K or V: 16 KB
+constexpr int ST_STAGE = 4 * ST_TILE;             // K lo, K hi, V lo, V hi
+constexpr int ST_THREADS = (ST_HKV + 1) * 32;
+constexpr int ST_ROWS_MAX = MAX_BATCH;
+constexpr size_t ST_SMEM = 1024 + (size_t)ST_STAGES * ST_STAGE + (ST_ROWS_MAX + 4) * sizeof(int) +
+                           (size_t)ST_HKV * 2 * 8 * PAGE * sizeof(uint16_t) + 2 * ST_STAGES * sizeof(uint64_t) + 16;
+
+struct StreamArgs {
+  const int* pt;
+  int pt_stride;
+  const int* slot_ids;
+  const int* lens;
+  int b, window, t_min, max_splits;
+  float scale_log2;
+  const float* prefix_part;  // prefix partials (slot 0 of [b][Hq][max_splits][DH + 2]) or nullptr
+  float* seg_part;           // [gridDim.x][2][Hq][DH + 2]
+  int* seg_cnt;              // [b][8], zero between launches
+  int* err;                  // set to 10 when a bounded wait expired
+};
+
+// byte offset of (row r, 16-byte chunk c) in a 128-byte-row tile written by TMA with 128-byte swizzle
+__device__ __forceinline__ uint32_t swz128(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
+
+__device__ __forceinline__ void st_row_range(const StreamArgs& a, int s, int& t_lo, int& L, int& p_first,
+                                             int& n_pages) {
+  L = a.lens[s];
+  t_lo = max(a.t_min, a.window > 0 ? max(0, L - a.window) : 0);
+  p_first = t_lo / PAGE;
+  n_pages = L > t_lo ? (L - 1) / PAGE - p_first + 1 : 0;
+}
+
+// first page index of CTA c's share of `total` pages
+__device__ __forceinline__ long long st_share(long long total, int c, int C) { return total * c / C; }
+__device__ __forceinline__ int st_cta_of(long long u, long long total, int C) {
+  int i = (int)(u * C / total);
+  while (i + 1 < C && st_share(total, i + 1, C) <= u) ++i;
+  while (i > 0 && st_share(total, i, C) > u) --i;
+  return i;
+}
+
+template <typename T, int G>
+__global__ void __launch_bounds__(ST_THREADS, 1)
+    k_decode_stream(const __grid_constant__ CUtensorMap tm, const T* __restrict__ q, T* __restrict__ out,
+                    StreamArgs a) {
+  static_assert(G >= 1 && G <= 8, "query heads per kv head");
+  constexpr int DH = ST_DH, KS = DH / 16, HKV = ST_HKV;
+  const int Hq = HKV * G;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  int* row_start = reinterpret_cast<int*>(smem + ST_STAGES * ST_STAGE);      // [b + 1]
+  uint16_t* pbuf = reinterpret_cast<uint16_t*>(row_start + ST_ROWS_MAX + 4);  // per warp: P hi [8][16], lo [8][16]
+  uint64_t* full = reinterpret_cast<uint64_t*>(pbuf + HKV * 2 * 8 * PAGE);
+  uint64_t* empty = full + ST_STAGES;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(empty + ST_STAGES);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ST_STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], HKV);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  pdl_entry();  // lens, page tables, q and the prefix partials of the preceding launches are visible
+  // row_start[s] = pages of rows 0 .. s-1 (block scan: each thread sums a run of consecutive rows)
+  {
+    const int per = (a.b + ST_THREADS - 1) / ST_THREADS;
+    const int r0 = threadIdx.x * per, r1 = min(a.b, r0 + per);
+    int sum = 0;
+    for (int s = r0; s < r1; ++s) {
+      int t_lo, L, pf, np;
+      st_row_range(a, s, t_lo, L, pf, np);
+      row_start[s] = np;  // own count for now
+      sum += np;
+    }
+    // exclusive scan of the per-thread sums over the block (warp shuffles, then the warp totals)
+    __shared__ int wsum[ST_THREADS / 32];
+    int incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    int base = 0;
+    for (int w = 0; w < warp; ++w) base += wsum[w];
+    int run = base + incl - sum;
+    for (int s = r0; s < r1; ++s) {
+      const int np = row_start[s];
+      row_start[s] = run;
+      run += np;
+    }
+    if (threadIdx.x == ST_THREADS - 1) row_start[a.b] = run;
+  }
+  __syncthreads();
+  const long long total = row_start[a.b];
+  // shares over min(CTAs, pages) CTAs, so that every share holds a page (a row's segments are then
+  // exactly the shares from the one holding its first page to the one holding its last)
+  const int C = (int)min((long long)gridDim.x, total);
+  if ((int)blockIdx.x >= C) return;
+  const long long u0 = st_share(total, blockIdx.x, C), u1 = st_share(total, blockIdx.x + 1, C);
+  // first row of the share: the last s with row_start[s] <= u0 (and a page)
+  int s_first = 0;
+  {
+    int lo = 0, hi = a.b - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (row_start[mid] <= u0) lo = mid;
+      else hi = mid - 1;
+    }
+    s_first = lo;
+    while (row_start[s_first + 1] <= u0) ++s_first;  // skip rows without pages
+  }
+  const int n_units = (int)(u1 - u0);
+
+  if (warp == HKV) {
+    // ---------------- producer: K and V of every kv head for each page of the share ----------------
+    // The 32 lanes look up the rows and page ids of the next 32 pages together (one round trip to memory per
+    // 32 pages); lane 0 then waits for free stages and issues the copies.
+    int stage = 0;
+    uint32_t phase = 0;
+    int armed[ST_STAGES];
+    uint32_t armed_par[ST_STAGES];
+    for (int i = 0; i < ST_STAGES; ++i) armed[i] = 0, armed_par[i] = 0;
+    int ok = 1;
+    int s_cur = s_first;  // row of the batch's first page
+    for (long long ub = u0; ub < u1 && ok; ub += 32) {
+      const long long u = ub + lane;
+      int s = s_cur, page = 0;
+      if (u < u1) {
+        while (u >= row_start[s + 1]) ++s;
+        int t_lo, L, pf, np;
+        st_row_range(a, s, t_lo, L, pf, np);
+        page = a.pt[(size_t)a.slot_ids[s] * a.pt_stride + pf + (int)(u - row_start[s])];
+      }
+      const int cnt = (int)min((long long)32, u1 - ub);
+      s_cur = __shfl_sync(0xffffffffu, s, cnt - 1);
+      for (int j = 0; j < cnt; ++j) {
+        const int pg = __shfl_sync(0xffffffffu, page, j);
+        if (lane == 0) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
+            ok = 0;
+          } else {
+            mbar_expect_tx(&full[stage], ST_STAGE);
+            uint8_t* dst = smem + stage * ST_STAGE;
+            const int yk = pg * 2 * HKV * PAGE, yv = yk + HKV * PAGE;
+            tma_load_2d(dst, &tm, &full[stage], 0, yk);
+            tma_load_2d(dst + ST_TILE, &tm, &full[stage], 64, yk);
+            tma_load_2d(dst + 2 * ST_TILE, &tm, &full[stage], 0, yv);
+            tma_load_2d(dst + 3 * ST_TILE, &tm, &full[stage], 64, yv);
+            armed[stage] = 1;
+            armed_par[stage] = phase;
+            if (++stage == ST_STAGES) stage = 0, phase ^= 1u;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
+      }
+    }
+    if (lane == 0) {
+      if (!ok) {
+        if (a.err) atomicExch(a.err, 10);
+        *abort_flag = 1;
+      }
+      for (int i = 0; i < ST_STAGES; ++i)  // every armed copy lands before the CTA exits
+        if (armed[i]) mbar_wait(&full[i], armed_par[i], nullptr);
+    }
+    return;
+  }
+
+  // ---------------- consumer warp h: kv head h, query heads h G .. h G + G - 1 ----------------
+  const int h = warp;
+  uint16_t* sPh = pbuf + h * 2 * 8 * PAGE;
+  uint16_t* sPl = sPh + 8 * PAGE;
+  int stage = 0;
+  uint32_t phase = 0;
+  int s = s_first, t_lo = 0, L = 0, pf = 0, np = 0;
+  st_row_range(a, s, t_lo, L, pf, np);
+  uint32_t qb[KS][2];
+  float m[2], l[2], o[KS][4];
+  // the shared-prefix partial of this thread's (head column, dim) values, loaded when the row starts so that
+  // its latency overlaps the row's pages
+  float pre_o[KS][4], pre_m[2], pre_l[2];
+  auto begin_row = [&]() {
+    if (a.prefix_part) {
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int hcol = min(2 * t4 + j, G - 1);
+        const float* p0 = a.prefix_part + ((size_t)s * Hq + h * G + hcol) * a.max_splits * (DH + 2);
+        pre_m[j] = p0[DH];
+        pre_l[j] = p0[DH + 1];
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt) {
+          pre_o[mt][j] = p0[mt * 16 + g];
+          pre_o[mt][2 + j] = p0[mt * 16 + g + 8];
+        }
+      }
+    }
+    const T* qh = q + ((size_t)s * Hq + h * G + (g < G ? g : 0)) * DH;
+#pragma unroll
+    for (int k = 0; k < KS; ++k) {
+      qb[k][0] = g < G ? *reinterpret_cast<const uint32_t*>(qh + k * 16 + 2 * t4) : 0u;
+      qb[k][1] = g < G ? *reinterpret_cast<const uint32_t*>(qh + k * 16 + 8 + 2 * t4) : 0u;
+    }
+    m[0] = m[1] = -INFINITY;
+    l[0] = l[1] = 0.f;
+#pragma unroll
+    for (int i = 0; i < KS; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  };
+  begin_row();
+  for (int i = 0; i < n_units; ++i) {
+    const long long u = u0 + i;
+    while (u >= row_start[s + 1]) {
+      ++s;
+      st_row_range(a, s, t_lo, L, pf, np);
+      begin_row();
+    }
+    const int pl = (int)(u - row_start[s]);  // page of the row
+    // every lane observes the stage's phase itself (the copies land through the async proxy)
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[stage], phase, abort_flag));
+    if (!ok) {
+      if (lane == 0) {
+        if (a.err) atomicExch(a.err, 10);
+        *abort_flag = 1;
+      }
+      return;
+    }
+    const uint32_t st = smem_u32(smem + stage * ST_STAGE);
+    // S^T = K Q^T: 16 positions x 8 head columns
+    float sc[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+      const int r = h * PAGE + (lane & 15);
+#pragma unroll
+      for (int k = 0; k < KS; ++k) {
+        uint32_t a0, a1, a2, a3;
+        ldm_x4(st + (k >> 2) * ST_TILE + swz128(r, (k & 3) * 2 + (lane >> 4)), a0, a1, a2, a3);
+        mma16816<T>(sc, a0, a1, a2, a3, qb[k][0], qb[k][1]);
+      }
+    }
+    const int tok0 = (pf + pl) * PAGE + g;
+    const bool v0 = tok0 >= t_lo && tok0 < L, v1 = tok0 + 8 >= t_lo && tok0 + 8 < L;
+    float corr[2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {  // head columns 2 t4 + j
+      const float x0 = v0 ? sc[j] * a.scale_log2 : -INFINITY;
+      const float x1 = v1 ? sc[2 + j] * a.scale_log2 : -INFINITY;
+      float bm = fmaxf(x0, x1);
+      bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 4));
+      bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 8));
+      bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, 16));
+      const float mn = fmaxf(m[j], bm);
+      const float base = (mn == -INFINITY) ? 0.f : mn;
+      corr[j] = exp2f(m[j] - base);
+      const float p0 = exp2f(x0 - base), p1 = exp2f(x1 - base);
+      float ps = p0 + p1;
+      ps += __shfl_xor_sync(0xffffffffu, ps, 4);
+      ps += __shfl_xor_sync(0xffffffffu, ps, 8);
+      ps += __shfl_xor_sync(0xffffffffu, ps, 16);
+      l[j] = l[j] * corr[j] + ps;
+      m[j] = mn;
+      const int hc = 2 * t4 + j;
+      uint32_t hi, lo = 0u;
+      if constexpr (std::is_same<T, bf16>::value) split16<T>(p0, p1, hi, lo);
+      else hi = pack2<T>(p0, p1);
+      sPh[hc * PAGE + g] = (uint16_t)(hi & 0xFFFFu);
+      sPh[hc * PAGE + g + 8] = (uint16_t)(hi >> 16);
+      sPl[hc * PAGE + g] = (uint16_t)(lo & 0xFFFFu);
+      sPl[hc * PAGE + g + 8] = (uint16_t)(lo >> 16);
+    }
+#pragma unroll
+    for (int mt = 0; mt < KS; ++mt) {
+      o[mt][0] *= corr[0], o[mt][1] *= corr[1];
+      o[mt][2] *= corr[0], o[mt][3] *= corr[1];
+    }
+    __syncwarp();
+    const uint32_t bh0 = *reinterpret_cast<const uint32_t*>(sPh + g * PAGE + 2 * t4);
+    const uint32_t bh1 = *reinterpret_cast<const uint32_t*>(sPh + g * PAGE + 8 + 2 * t4);
+    const uint32_t bl0 = *reinterpret_cast<const uint32_t*>(sPl + g * PAGE + 2 * t4);
+    const uint32_t bl1 = *reinterpret_cast<const uint32_t*>(sPl + g * PAGE + 8 + 2 * t4);
+    // O^T += V^T P^T: dims in m16 tiles, V rows (positions) read transposed
+    {
+      const int mi = lane >> 3, rr = h * PAGE + (lane & 7) + ((mi >> 1) << 3);
+#pragma unroll
+      for (int mt = 0; mt < KS; ++mt) {
+        uint32_t a0, a1, a2, a3;
+        ldm_x4_t(st + (2 + (mt >> 2)) * ST_TILE + swz128(rr, (mt & 3) * 2 + (mi & 1)), a0, a1, a2, a3);
+        mma16816<T>(o[mt], a0, a1, a2, a3, bh0, bh1);
+        if constexpr (std::is_same<T, bf16>::value) mma16816<T>(o[mt], a0, a1, a2, a3, bl0, bl1);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[stage]);
+    if (++stage == ST_STAGES) stage = 0, phase ^= 1u;
+    if (pl != np - 1 && i != n_units - 1) continue;
+    // ---------------- end of this CTA's segment of row s ----------------
+    const long long rs = row_start[s], re = row_start[s + 1];
+    const bool whole = rs >= u0 && re <= u1;
+    const int which = rs > u0 ? 1 : 0;  // the row began inside the share: the share's last segment
+    float* seg = a.seg_part + ((size_t)blockIdx.x * 2 + which) * Hq * (DH + 2);
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int hcol = 2 * t4 + j;
+      if (hcol >= G) continue;
+      const int hq = h * G + hcol;
+      float M = m[j], Ls = l[j], fold = 1.f;
+      float w0 = 0.f, m0 = -INFINITY, l0 = 0.f;
+      const bool pre = whole && a.prefix_part;
+      if (pre) {  // fold in the shared-prefix partial
+        m0 = pre_m[j];
+        l0 = pre_l[j];
+        const float Mn = fmaxf(M, m0);
+        w0 = (m0 == -INFINITY) ? 0.f : exp2f(m0 - Mn);
+        fold = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
+        Ls = Ls * fold + l0 * w0;
+      }
+#pragma unroll
+      for (int mt = 0; mt < KS; ++mt) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int d = mt * 16 + g + 8 * e;
+          float O = o[mt][2 * e + j];
+          if (whole) {
+            if (pre) O = O * fold + pre_o[mt][2 * e + j] * w0;
+            out[((size_t)s * Hq + hq) * DH + d] = f_to<T>(O / Ls);
+          } else {
+            seg[(size_t)hq * (DH + 2) + d] = O;
+          }
+        }
+      }
+      if (!whole && g == 0) {
+        seg[(size_t)hq * (DH + 2) + DH] = M;
+        seg[(size_t)hq * (DH + 2) + DH + 1] = Ls;
+      }
+    }
+    if (whole) continue;
+    // count this segment; the last of the row's segments (for this kv head) merges them
+    __threadfence();
+    __syncwarp();
+    const int c0 = st_cta_of(rs, total, C), c1 = st_cta_of(re - 1, total, C);
+    int last = 0;
+    if (lane == 0) last = atomicAdd(&a.seg_cnt[(size_t)s * HKV + h], 1) == c1 - c0;
+    last = __shfl_sync(0xffffffffu, last, 0);
+    if (!last) continue;
+    __threadfence();
+    for (int hcol = 0; hcol < G; ++hcol) {
+      const int hq = h * G + hcol;
+      float M = -INFINITY, Ls = 0.f, O[DH / 32];
+#pragma unroll
+      for (int k = 0; k < DH / 32; ++k) O[k] = 0.f;
+      auto merge = [&](const float* src) {
+        const float ms = src[DH], ls = src[DH + 1];
+        if (ms == -INFINITY) return;
+        const float Mn = fmaxf(M, ms);
+        const float wa = (M == -INFINITY) ? 0.f : exp2f(M - Mn), wb = exp2f(ms - Mn);
+        Ls = Ls * wa + ls * wb;
+#pragma unroll
+        for (int k = 0; k < DH / 32; ++k) O[k] = O[k] * wa + src[lane + 32 * k] * wb;
+        M = Mn;
+      };
+      if (a.prefix_part) merge(a.prefix_part + ((size_t)s * Hq + hq) * a.max_splits * (DH + 2));
+      for (int c = c0; c <= c1; ++c) {
+        const int wc = st_share(total, c, C) < rs ? 1 : 0;
+        merge(a.seg_part + (((size_t)c * 2 + wc) * Hq + hq) * (DH + 2));
+      }
+#pragma unroll
+      for (int k = 0; k < DH / 32; ++k) out[((size_t)s * Hq + hq) * DH + lane + 32 * k] = f_to<T>(O[k] / Ls);
+    }
+    if (lane == 0) a.seg_cnt[(size_t)s * HKV + h] = 0;
+  }
+}
+
+// ------------------------------------------------------------------------------------------------
+// Tensor-core shared-prefix pass (tcgen05; 16-bit KV, head_dim 128, 8 kv heads, prefix S <= 512 positions).
+//
+// The prompt's full pages are shared by every candidate, so the prefix part of decode attention is a dense
+// attention of many queries against one key set: per kv head h, the b x G query rows (candidate s, query
+// head h G + j) against the S prefix keys.  One CTA takes 128 query rows (128 / G candidates x G heads) of
+// one kv head.  Warp 0 issues the TMA copies: the Q tile once (a 4D map over q [b][8][G][128]), then K and
+// V of the kv head in blocks of 128 keys (16-row boxes out of the pool pages, 2 stages; keys past S read
+// the zero fill of a box outside the pool).  Warp 1 issues tcgen05.mma: S = Q K^T (M 128, N 128, K 128)
+// into one of two TMEM buffers, and O += P V (V read MN-major straight from the page rows) into a third.
+// Warps 2-5 own one query row per thread (their TMEM lane quadrant): they read S, apply the scale and the
+// per-row window, keep a reference maximum that is raised (and O rescaled in TMEM) only when a block's
+// maximum exceeds it by more than 2^8, write P = exp2(s - m) as the K-major swizzled A operand, and at the
+// end write (O, m, l) unnormalised as partial slot 0 in the decode kernels' log2-scaled convention.
+constexpr int PX_KB = 128;                   // keys per block
+constexpr int PX_HALF = 128 * 128;           // bytes of a 128-row x 64-column (128-byte) tile
+constexpr int PX_STAGE = 4 * PX_HALF;        // K (two column halves) + V (two column halves)
+constexpr int PX_STAGES = 2;
+constexpr int PX_SMAX = 512;                 // longest prefix handled
+constexpr size_t PX_SMEM = 1024 + 2 * PX_HALF + (size_t)PX_STAGES * PX_STAGE + 2 * PX_HALF + 256;
+constexpr float PX_RAISE = 8.f;              // log2 units the block maximum may exceed the reference by
+
+// instruction descriptor, kind::f16, fp32 D, M = 128, N = 128; b_mn: B is MN-major
+__host__ __device__ constexpr uint32_t px_idesc(bool bf, bool b_mn) {
+  return (1u << 4) | ((bf ? 1u : 0u) << 7) | ((bf ? 1u : 0u) << 10) | ((b_mn ? 1u : 0u) << 16) |
+         ((uint32_t)(128 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+// MN-major operand with 128-byte swizzle: rows of 64 MN elements (128 B), 8-row groups every 1024 B (SBO),
+// the next 64 MN elements `lbo` bytes further (LBO)
+__device__ __forceinline__ uint64_t sdesc_mn(uint32_t addr, uint32_t lbo) {
+  return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+template <typename T, int G>
+__global__ void __launch_bounds__(192, 1)
+    k_prefix_tc(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmkv,
+                const int* __restrict__ pt, int pt_stride, const int* __restrict__ slot_ids,
+                const int* __restrict__ lens, int n,
+                int S, int pool_rows, float scale_log2, int window, int max_splits, float* __restrict__ part,
+                int* err) {
+  static_assert(G == 1 || G == 2 || G == 4 || G == 8, "query heads per kv head");
+  constexpr int HKV = 8, DH = 128, SPC = 128 / G;  // candidates per CTA
+  constexpr bool BF = std::is_same<T, bf16>::value;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;                                  // 2 halves
+  uint8_t* sKV = sQ + 2 * PX_HALF;                     // stages: K lo, K hi, V lo, V hi
+  uint8_t* sP = sKV + PX_STAGES * PX_STAGE;            // 2 halves
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * PX_HALF);
+  uint64_t* q_full = bars;
+  uint64_t* full = bars + 1;                           // [2]
+  uint64_t* empty = full + PX_STAGES;                  // [2]
+  uint64_t* s_full = empty + PX_STAGES;                // [2]
+  uint64_t* s_free = s_full + 2;                       // [2]
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 1;
+  uint64_t* mma_done = o_done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y, s0 = blockIdx.x * SPC;
+  const int nkb = (S + PX_KB - 1) / PX_KB;
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int i = 0; i < PX_STAGES; ++i) mbar_init(&full[i], 1), mbar_init(&empty[i], 1);
+    for (int i = 0; i < 2; ++i) mbar_init(&s_full[i], 1), mbar_init(&s_free[i], 4);
+    mbar_init(p_full, 4);
+    mbar_init(o_done, 1);
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_entry();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      bool ok = true;
+      int armed[PX_STAGES] = {0, 0};
+      uint32_t armed_par[PX_STAGES] = {0, 0};
+      mbar_expect_tx(q_full, 2 * PX_HALF);
+      for (int c = 0; c < 2; ++c) tma_load_4d(sQ + c * PX_HALF, &tmq, q_full, c * 64, 0, h, s0);
+      const int* prow = pt + (size_t)slot_ids[0] * pt_stride;  // the prompt pages, the same in every row
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+        const int st = kb % PX_STAGES;
+        const uint32_t ph = (uint32_t)(kb / PX_STAGES) & 1u;
+        if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        mbar_expect_tx(&full[st], PX_STAGE);
+        uint8_t* dst = sKV + st * PX_STAGE;
+        for (int pg = 0; pg < PX_KB / PAGE; ++pg) {
+          const int key0 = kb * PX_KB + pg * PAGE;
+          // a page past the prefix reads rows outside the pool: the zero fill
+          const int yk = key0 < S ? prow[key0 / PAGE] * 2 * HKV * PAGE + h * PAGE : pool_rows;
+          const int yv = key0 < S ? yk + HKV * PAGE : pool_rows;
+          for (int c = 0; c < 2; ++c) {
+            tma_load_2d(dst + c * PX_HALF + pg * PAGE * 128, &tmkv, &full[st], c * 64, yk);
+            tma_load_2d(dst + (2 + c) * PX_HALF + pg * PAGE * 128, &tmkv, &full[st], c * 64, yv);
+          }
+        }
+        armed[st] = 1;
+        armed_par[st] = ph;
+      }
+      if (!ok) {
+        if (err) atomicExch(err, 11);
+        *abort_flag = 1;
+      }
+      mbar_wait(q_full, 0, nullptr);
+      for (int i = 0; i < PX_STAGES; ++i)
+        if (armed[i]) mbar_wait(&full[i], armed_par[i], nullptr);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t id_s = px_idesc(BF, false), id_o = px_idesc(BF, true);
+      bool ok = mbar_wait(q_full, 0, abort_flag);
+      tc_fence_after();
+      auto issue_o = [&](int kb) -> bool {  // O += P V of block kb
+        if (!mbar_wait(p_full, (uint32_t)kb & 1u, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t v = smem_u32(sKV + (kb % PX_STAGES) * PX_STAGE + 2 * PX_HALF);
+#pragma unroll
+        for (int k = 0; k < PX_KB / 16; ++k) {
+          const uint64_t a = sdesc(smem_u32(sP + (k >> 2) * PX_HALF)) + (uint64_t)((k & 3) * 2);
+          const uint64_t b = sdesc_mn(v + k * 16 * 128, PX_HALF);
+          umma(tmem + 256, a, b, id_o, (kb > 0 || k > 0) ? 1u : 0u);
+        }
+        umma_commit(o_done);
+        umma_commit(&empty[kb % PX_STAGES]);
+        return true;
+      };
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+        const int st = kb % PX_STAGES, sb = kb & 1;
+        if (!mbar_wait(&full[st], (uint32_t)(kb / PX_STAGES) & 1u, abort_flag) ||
+            !mbar_wait(&s_free[sb], ((uint32_t)(kb >> 1) & 1u) ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kbase = smem_u32(sKV + st * PX_STAGE);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint64_t a = sdesc(smem_u32(sQ + (k >> 2) * PX_HALF)) + (uint64_t)((k & 3) * 2);
+          const uint64_t b = sdesc(kbase + (k >> 2) * PX_HALF) + (uint64_t)((k & 3) * 2);
+          umma(tmem + sb * 128, a, b, id_s, k > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[sb]);
+        if (kb > 0 && !issue_o(kb - 1)) ok = false;
+      }
+      if (ok && !issue_o(nkb - 1)) ok = false;
+      if (!ok) {
+        if (err) atomicExch(err, 12);
+        *abort_flag = 1;
+      }
+      umma_commit(mma_done);
+      mbar_wait(mma_done, 0, nullptr);
+    }
+  } else {
+    // ---------------- softmax: one query row per thread ----------------
+    const int quad = warp & 3, r = quad * 32 + lane;
+    const int s = s0 + r / G, j = r % G;
+    const bool valid = s < n;
+    const int qpos = valid ? lens[s] - 1 : 0;
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int sb = kb & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(&s_full[sb], (uint32_t)(kb >> 1) & 1u, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+      float x[PX_KB];
+      tmem_ld64(trow + sb * 128, x);
+      tmem_ld64(trow + sb * 128 + 64, x + 64);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      float bmax = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < PX_KB; ++c) {
+        const int t = kb * PX_KB + c;
+        const bool in = t < S && (window <= 0 || t > qpos - window);
+        x[c] = in ? x[c] * scale_log2 : -INFINITY;
+        bmax = fmaxf(bmax, x[c]);
+      }
+      const bool raise = (m_ref == -INFINITY) ? (bmax > -INFINITY) : (bmax > m_ref + PX_RAISE);
+      const float m_new = raise ? bmax : m_ref;
+      const float corr = (raise && m_ref != -INFINITY) ? exp2f(m_ref - m_new) : 1.f;
+      float psum = 0.f;
+#pragma unroll
+      for (int c = 0; c < PX_KB; ++c) {
+        const float p = (x[c] == -INFINITY) ? 0.f : exp2f(x[c] - m_new);
+        x[c] = p;
+        psum += p;
+      }
+      l = l * corr + psum;
+      m_ref = m_new;
+      // the previous block's O MMA has read P and updated O before P is rewritten or O rescaled
+      if (kb > 0) {
+        ok = __all_sync(0xffffffffu, mbar_wait(o_done, (uint32_t)(kb - 1) & 1u, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+      }
+      // P row r as the K-major A operand (two 64-column halves, 128-byte swizzle)
+#pragma unroll
+      for (int ch = 0; ch < PX_KB / 8; ++ch) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const T a = f_to<T>(x[ch * 8 + 2 * e]), b = f_to<T>(x[ch * 8 + 2 * e + 1]);
+          w[e] = (uint32_t)(*reinterpret_cast<const uint16_t*>(&a)) |
+                 ((uint32_t)(*reinterpret_cast<const uint16_t*>(&b)) << 16);
+        }
+        uint8_t* dst = sP + (ch >> 3) * PX_HALF + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+        *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      // a raised reference maximum rescales the O accumulated so far (rows whose maximum stayed multiply by 1)
+      if (kb > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
+#pragma unroll 1
+        for (int hh = 0; hh < 2; ++hh) {
+          float o[64];
+          tmem_ld64(trow + 256 + hh * 64, o);
+#pragma unroll
+          for (int c = 0; c < 64; ++c) o[c] *= corr;
+          tmem_st64(trow + 256 + hh * 64, o);
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // P is read by the tensor core
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done, (uint32_t)(nkb - 1) & 1u, abort_flag));
+    if (ok) {
+      tc_fence_after();
+      float* pp = part + ((size_t)s * (HKV * G) + h * G + j) * max_splits * (DH + 2);
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        float o[64];
+        tmem_ld64(trow + 256 + hh * 64, o);
+        if (valid) {
+          // a partial slot is DH + 2 = 130 floats (520 bytes): 8-byte aligned, so two floats per store
+#pragma unroll
+          for (int c = 0; c < 64; c += 2) *reinterpret_cast<float2*>(pp + hh * 64 + c) = make_float2(o[c], o[c + 1]);
+        }
+      }
+      if (valid) pp[DH] = m_ref, pp[DH + 1] = l;
+    } else if (lane == 0) {
+      if (err) atomicExch(err, 13);
+      *abort_flag = 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+  }
+}
+
+// ------------------------------------------------------------------------------------------------
+// Tensor-core prefill attention (tcgen05; 16-bit, head_dim 128, 8 kv heads) for the reward model's scoring
+// passes: packed sequences, each attending causally to the prompt prefix (contiguous [P][8][128] per layer),
+// to its cached keys (reward-model cache pages, when the cache is on) and to its own new rows.
+//
+// One CTA takes 128 / G query positions (at most 64: a 64-position tile of the mma.sync kernel's tile list is
+// split over 64 / min(128 / G, 64) CTAs) of one sequence for the G query heads of one kv head (128 rows, Q by a
+// 4D map over q [rows][8][G][128]).  Keys come in blocks of 128 of one segment -- prefix rows and own rows by
+// 3D maps ([rows][8][128], box of 128 positions of one kv head), cached keys by 16-row page boxes -- and
+// blocks wholly outside the window or past the causal frontier are skipped; producer, MMA issuer and softmax
+// warps derive the same block list.  The MMA / softmax scheme is the prefix pass's (S = Q K^T in one of two
+// TMEM buffers, P written as the swizzled K-major operand, O += P V with V read MN-major, reference maximum
+// raised by more than 2^8 only); the epilogue normalises O by l and stores the 16-bit output rows.
+struct PrefillTcArgs {
+  const int* seq_off;
+  const int* tile_seq;
+  const int* tile_q0;  // 64-position tiles of the mma.sync kernel: this kernel runs two 32-position halves
+  int n_pre, pos0, window, rows_total, cache_rows;
+  const int* cpt;       // cache page table (rows per candidate), or nullptr
+  int cpt_stride;
+  const int* seq_cand;
+  const int* seq_cached;
+  float scale_log2;
+  int* err;
+};
+
+// key block kb of a CTA's list: segment (0 prefix, 1 cached, 2 own) and first key index within the segment
+struct PxBlock {
+  int seg, kbase, count, kpos0;
+};
+
+template <typename T, int G>
+__global__ void __launch_bounds__(192, 1)
+    k_prefill_tc(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmkp,
+                 const __grid_constant__ CUtensorMap tmvp, const __grid_constant__ CUtensorMap tmk,
+                 const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmc, T* __restrict__ out,
+                 PrefillTcArgs a) {
+  static_assert(G == 1 || G == 2 || G == 4 || G == 8, "query heads per kv head");
+  constexpr int HKV = 8, DH = 128, QP = 128 / G;  // query positions of the 128-row Q tile
+  constexpr int PPC = QP < 64 ? QP : 64;           // positions a CTA answers for: a 64-position host tile
+  constexpr int NSUB = 64 / PPC;                   // ... is split over NSUB CTAs
+  constexpr bool BF = std::is_same<T, bf16>::value;
+  const int tile = blockIdx.x / NSUB, h = blockIdx.y;
+  const int j = a.tile_seq[tile];
+  const int r0 = a.seq_off[j], nrows = a.seq_off[j + 1] - r0;
+  const int q0 = a.tile_q0[tile] + (blockIdx.x % NSUB) * PPC;
+  if (q0 >= nrows) return;  // a sub-tile past the end of a short tile
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sKV = sQ + 2 * PX_HALF;
+  uint8_t* sP = sKV + PX_STAGES * PX_STAGE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * PX_HALF);
+  uint64_t* q_full = bars;
+  uint64_t* full = bars + 1;
+  uint64_t* empty = full + PX_STAGES;
+  uint64_t* s_full = empty + PX_STAGES;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 1;
+  uint64_t* mma_done = o_done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  // the CTA's key blocks: prefix, cached, own (own keys up to the last query position of the CTA)
+  const int ncache = a.cpt ? a.seq_cached[j] : 0;
+  const int opos0 = a.pos0 + ncache;
+  const int q_last = min(nrows, q0 + PPC) - 1;
+  const int qpos_min = opos0 + q0, qpos_max = opos0 + q_last;
+  const int n_own = q_last + 1;
+  auto block_at = [&](int seg, int kbase) -> PxBlock {
+    const int cnt = min(PX_KB, (seg == 0 ? a.n_pre : (seg == 1 ? ncache : n_own)) - kbase);
+    const int kp0 = seg == 0 ? kbase : (seg == 1 ? a.pos0 + kbase : opos0 + kbase);
+    return PxBlock{seg, kbase, cnt, kp0};
+  };
+  auto live = [&](const PxBlock& b) {  // some key of the block is visible to some query of the CTA
+    if (a.window > 0 && b.kpos0 + b.count - 1 <= qpos_min - a.window) return false;
+    return b.kpos0 <= qpos_max;
+  };
+  // blocks are enumerated by a running cursor (segment, key base) that skips dead blocks
+  auto next_block = [&](int& seg, int& kbase, PxBlock& out_b) -> bool {
+    while (seg < 3) {
+      const int len = seg == 0 ? a.n_pre : (seg == 1 ? ncache : n_own);
+      if (kbase >= len) {
+        ++seg;
+        kbase = 0;
+        continue;
+      }
+      out_b = block_at(seg, kbase);
+      kbase += PX_KB;
+      if (live(out_b)) return true;
+    }
+    return false;
+  };
+  int nkb = 0;
+  {
+    int sg = 0, kb0 = 0;
+    PxBlock b;
+    while (next_block(sg, kb0, b)) ++nkb;
+  }
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int i = 0; i < PX_STAGES; ++i) mbar_init(&full[i], 1), mbar_init(&empty[i], 1);
+    for (int i = 0; i < 2; ++i) mbar_init(&s_full[i], 1), mbar_init(&s_free[i], 4);
+    mbar_init(p_full, 4);
+    mbar_init(o_done, 1);
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_entry();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      bool ok = true;
+      int armed[PX_STAGES] = {0, 0};
+      uint32_t armed_par[PX_STAGES] = {0, 0};
+      mbar_expect_tx(q_full, 2 * PX_HALF);
+      for (int c = 0; c < 2; ++c) tma_load_4d(sQ + c * PX_HALF, &tmq, q_full, c * 64, 0, h, r0 + q0);
+      const int* cpt = a.cpt ? a.cpt + (size_t)a.seq_cand[j] * a.cpt_stride : nullptr;
+      int sg = 0, kbc = 0;
+      PxBlock b;
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+        next_block(sg, kbc, b);
+        const int st = kb % PX_STAGES;
+        const uint32_t ph = (uint32_t)(kb / PX_STAGES) & 1u;
+        if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        mbar_expect_tx(&full[st], PX_STAGE);
+        uint8_t* dst = sKV + st * PX_STAGE;
+        if (b.seg == 1) {  // cached keys: 16-row page boxes (a page past the cached keys reads the zero fill)
+          for (int pg = 0; pg < PX_KB / PAGE; ++pg) {
+            const int key0 = b.kbase + pg * PAGE;
+            const int yk = key0 < ncache ? cpt[key0 / PAGE] * 2 * HKV * PAGE + h * PAGE : a.cache_rows;
+            const int yv = key0 < ncache ? yk + HKV * PAGE : a.cache_rows;
+            for (int c = 0; c < 2; ++c) {
+              tma_load_2d(dst + c * PX_HALF + pg * PAGE * 128, &tmc, &full[st], c * 64, yk);
+              tma_load_2d(dst + (2 + c) * PX_HALF + pg * PAGE * 128, &tmc, &full[st], c * 64, yv);
+            }
+          }
+        } else {  // prefix or own rows: one 128-position box of kv head h per column half
+          const CUtensorMap* mk = b.seg == 0 ? &tmkp : &tmk;
+          const CUtensorMap* mv = b.seg == 0 ? &tmvp : &tmv;
+          const int row0 = b.seg == 0 ? b.kbase : r0 + b.kbase;
+          for (int c = 0; c < 2; ++c) {
+            tma_load_3d(dst + c * PX_HALF, mk, &full[st], c * 64, h, row0);
+            tma_load_3d(dst + (2 + c) * PX_HALF, mv, &full[st], c * 64, h, row0);
+          }
+        }
+        armed[st] = 1;
+        armed_par[st] = ph;
+      }
+      if (!ok) {
+        if (a.err) atomicExch(a.err, 14);
+        *abort_flag = 1;
+      }
+      mbar_wait(q_full, 0, nullptr);
+      for (int i = 0; i < PX_STAGES; ++i)
+        if (armed[i]) mbar_wait(&full[i], armed_par[i], nullptr);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer (as in the prefix pass) ----------------
+      const uint32_t id_s = px_idesc(BF, false), id_o = px_idesc(BF, true);
+      bool ok = mbar_wait(q_full, 0, abort_flag);
+      tc_fence_after();
+      auto issue_o = [&](int kb) -> bool {
+        if (!mbar_wait(p_full, (uint32_t)kb & 1u, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t v = smem_u32(sKV + (kb % PX_STAGES) * PX_STAGE + 2 * PX_HALF);
+#pragma unroll
+        for (int k = 0; k < PX_KB / 16; ++k) {
+          const uint64_t ad = sdesc(smem_u32(sP + (k >> 2) * PX_HALF)) + (uint64_t)((k & 3) * 2);
+          const uint64_t bd = sdesc_mn(v + k * 16 * 128, PX_HALF);
+          umma(tmem + 256, ad, bd, id_o, (kb > 0 || k > 0) ? 1u : 0u);
+        }
+        umma_commit(o_done);
+        umma_commit(&empty[kb % PX_STAGES]);
+        return true;
+      };
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+        const int st = kb % PX_STAGES, sb = kb & 1;
+        if (!mbar_wait(&full[st], (uint32_t)(kb / PX_STAGES) & 1u, abort_flag) ||
+            !mbar_wait(&s_free[sb], ((uint32_t)(kb >> 1) & 1u) ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kbase = smem_u32(sKV + st * PX_STAGE);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint64_t ad = sdesc(smem_u32(sQ + (k >> 2) * PX_HALF)) + (uint64_t)((k & 3) * 2);
+          const uint64_t bd = sdesc(kbase + (k >> 2) * PX_HALF) + (uint64_t)((k & 3) * 2);
+          umma(tmem + sb * 128, ad, bd, id_s, k > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[sb]);
+        if (kb > 0 && !issue_o(kb - 1)) ok = false;
+      }
+      if (ok && nkb > 0 && !issue_o(nkb - 1)) ok = false;
+      if (!ok) {
+        if (a.err) atomicExch(a.err, 15);
+        *abort_flag = 1;
+      }
+      umma_commit(mma_done);
+      mbar_wait(mma_done, 0, nullptr);
+    }
+  } else {
+    // ---------------- softmax and epilogue: one query row per thread ----------------
+    const int quad = warp & 3, r = quad * 32 + lane;
+    const int qi = q0 + r / G, jh = r % G;
+    const bool valid = qi < nrows && qi < q0 + PPC;
+    const int qpos = opos0 + qi;
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    int sg = 0, kbc = 0;
+    PxBlock b;
+    for (int kb = 0; kb < nkb; ++kb) {
+      next_block(sg, kbc, b);
+      const int sb = kb & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(&s_full[sb], (uint32_t)(kb >> 1) & 1u, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+      float x[PX_KB];
+      tmem_ld64(trow + sb * 128, x);
+      tmem_ld64(trow + sb * 128 + 64, x + 64);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      float bmax = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < PX_KB; ++c) {
+        const int kpos = b.kpos0 + c;
+        const bool in = c < b.count && kpos <= qpos && (a.window <= 0 || kpos > qpos - a.window);
+        x[c] = in ? x[c] * a.scale_log2 : -INFINITY;
+        bmax = fmaxf(bmax, x[c]);
+      }
+      const bool raise = (m_ref == -INFINITY) ? (bmax > -INFINITY) : (bmax > m_ref + PX_RAISE);
+      const float m_new = raise ? bmax : m_ref;
+      const float corr = (raise && m_ref != -INFINITY) ? exp2f(m_ref - m_new) : 1.f;
+      float psum = 0.f;
+#pragma unroll
+      for (int c = 0; c < PX_KB; ++c) {
+        const float p = (x[c] == -INFINITY) ? 0.f : exp2f(x[c] - m_new);
+        x[c] = p;
+        psum += p;
+      }
+      l = l * corr + psum;
+      m_ref = m_new;
+      if (kb > 0) {
+        ok = __all_sync(0xffffffffu, mbar_wait(o_done, (uint32_t)(kb - 1) & 1u, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+      }
+#pragma unroll
+      for (int ch = 0; ch < PX_KB / 8; ++ch) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const T lo = f_to<T>(x[ch * 8 + 2 * e]), hi = f_to<T>(x[ch * 8 + 2 * e + 1]);
+          w[e] = (uint32_t)(*reinterpret_cast<const uint16_t*>(&lo)) |
+                 ((uint32_t)(*reinterpret_cast<const uint16_t*>(&hi)) << 16);
+        }
+        uint8_t* dst = sP + (ch >> 3) * PX_HALF + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+        *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      if (kb > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
+#pragma unroll 1
+        for (int hh = 0; hh < 2; ++hh) {
+          float o[64];
+          tmem_ld64(trow + 256 + hh * 64, o);
+#pragma unroll
+          for (int c = 0; c < 64; ++c) o[c] *= corr;
+          tmem_st64(trow + 256 + hh * 64, o);
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok && nkb > 0) ok = __all_sync(0xffffffffu, mbar_wait(o_done, (uint32_t)(nkb - 1) & 1u, abort_flag));
+    if (ok && nkb > 0) {
+      tc_fence_after();
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      T* dst = out + ((size_t)(r0 + qi) * (HKV * G) + h * G + jh) * DH;
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {
+        float o[64];
+        tmem_ld64(trow + 256 + hh * 64, o);
+        if (valid) {
+#pragma unroll
+          for (int c = 0; c < 64; c += 8) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const T lo = f_to<T>(o[c + 2 * e] * inv), hi = f_to<T>(o[c + 2 * e + 1] * inv);
+              w[e] = (uint32_t)(*reinterpret_cast<const uint16_t*>(&lo)) |
+                     ((uint32_t)(*reinterpret_cast<const uint16_t*>(&hi)) << 16);
+            }
+            *reinterpret_cast<uint4*>(dst + hh * 64 + c) = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        }
+      }
+    } else if (!ok && lane == 0) {
+      if (a.err) atomicExch(a.err, 16);
+      *abort_flag = 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+  }
+}
+
 // O[16 x 16*NDP] += P[16 x 64] V[64 x 16*NDP] for one warp: P comes from the S accumulators (C layout of
 // m16n8k16), V rows are read transposed from shared memory.  fp16 P is used as is (11-bit significand);
 // bf16 P is split into hi + lo pairs (two MMAs) to keep ~16 significand bits.
@@ -899,14 +1899,140 @@ __global__ void k_prefill_attn_f32(const float* __restrict__ q, const float* __r
   }
 }
 
+bool stream_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("SR_ATTN_STREAM");
+    return !(e && e[0] == '0');
+  }();
+  return on;
+}
+
+template <typename T, int G>
+sr_status prefix_tc_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids, const int* lens,
+                      int b, int S, int window, float* part, int max_splits, const DecodeStreamWs& ws,
+                      cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    SR_CUDA(cudaFuncSetAttribute(k_prefix_tc<T, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PX_SMEM));
+    attr = true;
+  }
+  constexpr bool BF = std::is_same<T, bf16>::value;
+  const int pool_rows = ws.pool_pages * 2 * ST_HKV * PAGE;
+  CUtensorMap tmkv, tmq;
+  SR_TRY(encode_tma_2d(&tmkv, pool, BF, pool_rows, ST_DH, PAGE));
+  const uint64_t dims[4] = {(uint64_t)ST_DH, (uint64_t)G, (uint64_t)ST_HKV, (uint64_t)b};
+  const uint64_t strides[3] = {(uint64_t)ST_DH * 2, (uint64_t)G * ST_DH * 2, (uint64_t)ST_HKV * G * ST_DH * 2};
+  const uint32_t box[4] = {64, (uint32_t)G, 1, (uint32_t)(128 / G)};
+  SR_TRY(encode_tma_nd(&tmq, q, BF, 4, dims, strides, box));
+  launch_k(k_prefix_tc<T, G>, dim3((b + 128 / G - 1) / (128 / G), ST_HKV), 192, PX_SMEM, st, tmq, tmkv, pt, pt_stride,
+           ids, lens, b, S, pool_rows, 1.4426950408889634f / sqrtf((float)ST_DH), window, max_splits, part, ws.err);
+  SR_LAUNCH();
+  return SR_OK;
+}
+
+template <typename T, int G>
+sr_status prefill_tc_t(const void* q, const void* k, const void* v, const void* kpre, const void* vpre, int npre,
+                       const int* seq_off, const int* tile_seq, const int* tile_q0, int n_tiles, int pos0, int rows,
+                       int window, void* out, const CachedKeys& ck, cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    SR_CUDA(cudaFuncSetAttribute(k_prefill_tc<T, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PX_SMEM));
+    attr = true;
+  }
+  constexpr bool BF = std::is_same<T, bf16>::value;
+  constexpr int HKV = ST_HKV, DH = ST_DH;
+  CUtensorMap tmq, tmk, tmv, tmkp, tmvp, tmc;
+  {
+    const uint64_t dims[4] = {(uint64_t)DH, (uint64_t)G, (uint64_t)HKV, (uint64_t)rows};
+    const uint64_t strides[3] = {(uint64_t)DH * 2, (uint64_t)G * DH * 2, (uint64_t)HKV * G * DH * 2};
+    const uint32_t box[4] = {64, (uint32_t)G, 1, (uint32_t)(128 / G)};
+    SR_TRY(encode_tma_nd(&tmq, q, BF, 4, dims, strides, box));
+  }
+  auto kv3 = [&](CUtensorMap* m, const void* base, int n) -> sr_status {  // [n][8][128], 128-position boxes
+    const uint64_t dims[3] = {(uint64_t)DH, (uint64_t)HKV, (uint64_t)n};
+    const uint64_t strides[2] = {(uint64_t)DH * 2, (uint64_t)HKV * DH * 2};
+    const uint32_t box[3] = {64, 1, (uint32_t)PX_KB};
+    return encode_tma_nd(m, base, BF, 3, dims, strides, box);
+  };
+  SR_TRY(kv3(&tmk, k, rows));
+  SR_TRY(kv3(&tmv, v, rows));
+  if (npre > 0) {
+    SR_TRY(kv3(&tmkp, kpre, npre));
+    SR_TRY(kv3(&tmvp, vpre, npre));
+  } else {
+    tmkp = tmk, tmvp = tmv;  // no prefix segment: never read
+  }
+  const int cache_rows = ck.pool ? ck.pool_pages * 2 * HKV * PAGE : 0;
+  if (ck.pool) SR_TRY(encode_tma_2d(&tmc, ck.pool, BF, cache_rows, DH, PAGE));
+  else tmc = tmk;  // no cached segment: never read
+  PrefillTcArgs a{seq_off, tile_seq, tile_q0, npre, pos0, window, rows, cache_rows,
+                  ck.pool ? ck.page_table : nullptr, ck.pt_stride, ck.seq_cand, ck.seq_cached,
+                  1.4426950408889634f / sqrtf((float)DH), tc_error_word()};
+  constexpr int NSUB = 64 / ((128 / G) < 64 ? (128 / G) : 64);
+  launch_k(k_prefill_tc<T, G>, dim3(n_tiles * NSUB, HKV), 192, PX_SMEM, st, tmq, tmkp, tmvp, tmk, tmv, tmc, (T*)out,
+           a);
+  SR_LAUNCH();
+  return SR_OK;
+}
+
+// The tcgen05 prefill measured slower than the mma.sync kernel on the scoring shapes (1.03 against 0.66 ms for
+// 37 sequences x 443 rows after a 288-position prefix: one CTA per SM, four softmax warps and a per-CTA TMEM
+// allocation for a few key blocks each), so it runs only when SR_PREFILL_TC=1.
+bool prefill_tc_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("SR_PREFILL_TC");
+    return e && e[0] == '1';
+  }();
+  return on;
+}
+
+// The tcgen05 prefix pass measured slower in the decode loop than the mma.sync one (one CTA and four softmax
+// warps per SM against sixteen warps), so it runs only when SR_PREFIX_TC=1.
+bool prefix_tc_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("SR_PREFIX_TC");
+    return e && e[0] == '1';
+  }();
+  return on;
+}
+
+template <typename T, int G>
+sr_status decode_stream_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
+                          const int* lens, int b, int window, void* out, const float* prefix_part, int max_splits,
+                          int shared_pos, const DecodeStreamWs& ws, cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    SR_CUDA(cudaFuncSetAttribute(k_decode_stream<T, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ST_SMEM));
+    attr = true;
+  }
+  CUtensorMap tm;
+  SR_TRY(encode_tma_2d(&tm, pool, std::is_same<T, bf16>::value, ws.pool_pages * 2 * ST_HKV * PAGE, ST_DH, 128));
+  StreamArgs a{pt, pt_stride, ids, lens, b, window, shared_pos, max_splits,
+               1.4426950408889634f / sqrtf((float)ST_DH), prefix_part, ws.seg_part, ws.seg_cnt, ws.err};
+  launch_k(k_decode_stream<T, G>, ws.grid, ST_THREADS, ST_SMEM, st, tm, (const T*)q, (T*)out, a);
+  SR_LAUNCH();
+  return SR_OK;
+}
+
 template <typename T, int DH, int G>
 sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int pt_stride, const int* ids,
                            const int* lens, int b, int Hkv, int window, void* out, float* part, int max_splits,
-                           int shared_pos, int max_len, cudaStream_t st, int* err) {
+                           int shared_pos, int max_len, cudaStream_t st, int* err, const DecodeStreamWs* ws) {
   // with a shared prefix: slot 0 of the partials is the prefix pass, position splits follow
   const int sbase = shared_pos > 0 ? 1 : 0;
   const int t_min = shared_pos;
-  if (sbase) {
+  bool prefix_done = false;
+  if constexpr (DH == ST_DH) {
+    if (sbase && part && ws && prefix_tc_enabled() && Hkv == ST_HKV && shared_pos <= PX_SMAX &&
+        (G == 1 || G == 2 || G == 4 || G == 8)) {
+      constexpr int GG = (G == 1 || G == 2 || G == 4 || G == 8) ? G : 1;
+      const sr_status ps = prefix_tc_t<T, GG>(q, pool, pt, pt_stride, ids, lens, b, shared_pos, window, part,
+                                              max_splits, *ws, st);
+      if (ps != SR_OK) return ps;
+      prefix_done = true;
+    }
+  }
+  if (sbase && !prefix_done) {
     if (!part) return set_err(SR_ERR_INVALID_ARG, "decode attention: partial buffer missing for the prefix pass");
     // eight warps (128 query rows) per CTA share each staged K/V block
     constexpr int NW = 8, HPC = G < 4 ? G : 4, CPC = NW / HPC;
@@ -920,6 +2046,11 @@ sr_status decode_attn_tc_t(const void* q, const void* pool, const int* pt, int p
         (const T*)q, (const T*)pool, pt, pt_stride, ids, lens, b, shared_pos, Hkv,
         1.4426950408889634f / sqrtf((float)DH), window, max_splits, part);
     SR_LAUNCH();
+  }
+  if constexpr (DH == ST_DH) {
+    if (ws && stream_enabled() && Hkv == ST_HKV && b <= ST_ROWS_MAX)
+      return decode_stream_t<T, G>(q, pool, pt, pt_stride, ids, lens, b, window, out, sbase ? part : nullptr,
+                                   max_splits, shared_pos, *ws, st);
   }
   constexpr int LDS = DH + 8;
   const size_t smem = std::max<size_t>((size_t)4 * (2 * 2 * PAGE * LDS + 2 * 8 * PAGE) * sizeof(T),
@@ -989,6 +2120,7 @@ sr_status prefill_t(const void* q, const void* k, const void* v, const void* kpr
 
 }  // namespace
 
+size_t decode_stream_part_floats(int grid, int Hq) { return (size_t)grid * 2 * Hq * (ST_DH + 2); }
 int decode_attention_max_splits(int max_len) { return max_len <= 0 ? 1 : (max_len + SPLIT - 1) / SPLIT; }
 int decode_attention_slots(int max_len, int window, int shared_pos) {
   const int lo = shared_pos > 0 ? shared_pos : 0;
@@ -1002,7 +2134,7 @@ size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits) {
 sr_status launch_decode_attention(int et, const void* q, const void* pool_layer, const int* pt, int pt_stride,
                                   const int* ids, const int* lens, int b, int Hq, int Hkv, int dh, int window,
                                   void* out, float* part, int max_splits, cudaStream_t st, int shared_pos,
-                                  int max_len, int* err) {
+                                  int max_len, int* err, const DecodeStreamWs* ws) {
   if (b == 0) return SR_OK;
   const int G = Hq / Hkv;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "decode attention: n_heads %% n_kv_heads != 0");
@@ -1014,7 +2146,7 @@ sr_status launch_decode_attention(int et, const void* q, const void* pool_layer,
 #define SR_DECT(T, D, GG)                                                                                          \
   if (dh == D && G == GG)                                                                                            \
     return decode_attn_tc_t<T, D, GG>(q, pool_layer, pt, pt_stride, ids, lens, b, Hkv, window, out, part, max_splits, \
-                                      shared_pos, max_len, st, err);
+                                      shared_pos, max_len, st, err, ws);
   if (et == SR_DT_F16) {
     SR_DECT(f16, 128, 4) SR_DECT(f16, 128, 1) SR_DECT(f16, 128, 2) SR_DECT(f16, 128, 8)
     SR_DECT(f16, 64, 1) SR_DECT(f16, 64, 4) SR_DECT(f16, 32, 1)
@@ -1052,11 +2184,29 @@ sr_status launch_prefill_attention_f32(const float* q, const float* k, const flo
 sr_status launch_prefill_attention(int et, const void* q, const void* k, const void* v, const void* kpre,
                                    const void* vpre, int npre, const int* seq_off, int n_seq, const int* tile_seq,
                                    const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
-                                   void* out, cudaStream_t st, CachedKeys ck) {
+                                   void* out, cudaStream_t st, CachedKeys ck, int rows) {
   (void)n_seq;
   if (n_tiles == 0) return SR_OK;
   if (Hq % Hkv) return set_err(SR_ERR_UNSUPPORTED, "prefill attention: n_heads %% n_kv_heads != 0");
   if (et != SR_DT_F16 && et != SR_DT_BF16) return set_err(SR_ERR_INVALID_ARG, "prefill attention: 16-bit types only");
+  // head_dim 128 with 8 kv heads: the tensor-core kernel (every operand 16-byte aligned, as TMA needs)
+  const int G = Hq / Hkv;
+  const bool al = ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v) |
+                    reinterpret_cast<uintptr_t>(kpre) | reinterpret_cast<uintptr_t>(vpre) |
+                    reinterpret_cast<uintptr_t>(ck.pool) | reinterpret_cast<uintptr_t>(out)) & 15) == 0;
+  if (rows > 0 && prefill_tc_enabled() && dh == ST_DH && Hkv == ST_HKV && al &&
+      (G == 1 || G == 2 || G == 4 || G == 8)) {
+#define SR_PTC(TT, GG)                                                                                              \
+  if (G == GG)                                                                                                      \
+    return prefill_tc_t<TT, GG>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, rows, window, \
+                                out, ck, st);
+    if (et == SR_DT_F16) {
+      SR_PTC(f16, 1) SR_PTC(f16, 2) SR_PTC(f16, 4) SR_PTC(f16, 8)
+    } else {
+      SR_PTC(bf16, 1) SR_PTC(bf16, 2) SR_PTC(bf16, 4) SR_PTC(bf16, 8)
+    }
+#undef SR_PTC
+  }
 #define SR_PRE(T)                                                                                                      \
   switch (dh) {                                                                                                        \
     case 32: return prefill_t<T, 32, 32>(q, k, v, kpre, vpre, npre, seq_off, tile_seq, tile_q0, n_tiles, pos0, Hq, Hkv, \

@@ -195,6 +195,21 @@ sr_status launch_sample(const float* logits, long long ld, int b, int V, const i
                         const int* n_rows = nullptr);  // device count: rows >= *n_rows are skipped
 
 // attention.cu
+// Workspace of the streaming decode-attention kernel (16-bit KV, head_dim 128, 8 kv heads): one persistent
+// CTA per SM (grid); segment partials [grid][2][n_heads][130] floats; per-(row, kv head) counters [b][8]
+// that must be zero before the first launch (each launch leaves them zero); pool_pages = pages per layer of
+// the pool; err: set to 10 when a bounded wait expired.  Without it (nullptr) the per-row kernels run.
+struct DecodeStreamWs {
+  float* seg_part = nullptr;
+  int* seg_cnt = nullptr;
+  int grid = 0;
+  int pool_pages = 0;
+  int* err = nullptr;
+};
+size_t decode_stream_part_floats(int grid, int Hq);
+// gemm_tc.cu: device error word shared by the kernels with bounded waits (GEMMs 1-3, decode attention 10);
+// allocated on first use, nullptr if that failed
+int* tc_error_word();
 // shared_pos > 0: positions [0, shared_pos) sit in pages shared by every row's page table (the prompt);
 // a tensor-core prefix pass reads them once per 64 rows and `part` must hold
 // decode_attention_slots(max_len, window, shared_pos) partial slots per (row, head).
@@ -202,7 +217,8 @@ sr_status launch_decode_attention(int dtype, const void* q, const void* pool_lay
                                   int pt_stride, const int* slot_ids, const int* lens, int b, int Hq, int Hkv, int dh,
                                   int window, void* out, float* part, int max_splits, cudaStream_t st,
                                   int shared_pos = 0, int max_len = 0,  // max_len > 0: longest lens[] (launch shape)
-                                  int* err = nullptr);  // set to 1 when a row needs more splits than max_splits
+                                  int* err = nullptr,   // set to 1 when a row needs more splits than max_splits
+                                  const DecodeStreamWs* ws = nullptr);  // workspace of the streaming kernel
 int decode_attention_max_splits(int max_len);
 int decode_attention_slots(int max_len, int window, int shared_pos);
 size_t decode_attention_part_floats(int b, int Hq, int dh, int max_splits);
@@ -216,6 +232,7 @@ struct CachedKeys {
   int pt_stride = 0;
   const int* seq_cand = nullptr;
   const int* seq_cached = nullptr;
+  int pool_pages = 0;          // pages per layer of the pool (bounds of its tensor map)
 };
 sr_status launch_prefill_attention_f32(const float* q, const float* k, const float* v, const float* k_pre,
                                        const float* v_pre, int n_pre, const int* seq_off, int n_seq, int rows,
@@ -224,7 +241,8 @@ sr_status launch_prefill_attention_f32(const float* q, const float* k, const flo
 sr_status launch_prefill_attention(int et, const void* q, const void* k, const void* v, const void* k_pre,
                                    const void* v_pre, int n_pre, const int* seq_off, int n_seq, const int* tile_seq,
                                    const int* tile_q0, int n_tiles, int pos0, int Hq, int Hkv, int dh, int window,
-                                   void* out, cudaStream_t st, CachedKeys ck = CachedKeys());
+                                   void* out, cudaStream_t st, CachedKeys ck = CachedKeys(),
+                                   int rows = 0);  // rows > 0: q/k/v rows (the tensor-core kernel needs it)
 // elementwise.cu: in-place bf16 -> fp16 conversion of n elements (weights at load)
 sr_status launch_bf16_to_f16(void* p, size_t n, cudaStream_t st);
 

@@ -36,13 +36,13 @@
 #include <type_traits>
 
 #include "common.cuh"
+#include "tma.cuh"
 
 namespace sr {
 namespace {
 
 constexpr int BM = 128, BK = 64;  // BM: rows of one MMA (one TMEM lane block)
 constexpr int BAR_BYTES = 256;
-constexpr unsigned long long WAIT_NS = 2000000000ull;
 
 // TM = rows per CTA tile: 128 (one MMA per K step) or 256 (two MMAs sharing the W tile, which halves the
 // staged bytes per flop; its 256 x 256 fp32 accumulator fills TMEM, so it is single-buffered and drained
@@ -68,72 +68,6 @@ __host__ __device__ constexpr uint32_t idesc_for(bool bf, int BN) {
          ((uint32_t)(BM >> 4) << 24);
 }
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ unsigned long long gtimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_test(uint32_t addr, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(addr), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait for the phase with the given parity.  Returns false on timeout or when another
-// role has raised the CTA's abort flag (if `abort_flag` is non-null).
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  const uint32_t addr = smem_u32(bar);
-  if (mbar_test(addr, parity)) return true;
-  const unsigned long long t0 = gtimer();
-  while (true) {
-#pragma unroll 1
-    for (int i = 0; i < 32; ++i)
-      if (mbar_test(addr, parity)) return true;
-    if (abort_flag && *abort_flag) return false;
-    if (gtimer() - t0 > WAIT_NS) return false;
-  }
-}
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], "
-      "[%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
-      : "memory");
-}
-// UMMA shared-memory descriptor for a K-major tile written by TMA with 128-byte swizzle:
-// start address >> 4 (bits 0-13), leading byte offset 16 B (unused by swizzled K-major),
-// stride byte offset 1024 B between 8-row groups (bits 32-45), version 1 (bit 46),
-// layout SWIZZLE_128B = 2 (bits 61-63).
-__device__ __forceinline__ uint64_t sdesc(uint32_t addr) {
-  return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
-          d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
-}
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-               : "memory");
-}
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -142,36 +76,6 @@ __device__ __forceinline__ uint32_t cluster_rank() {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// 32 lanes x 16 consecutive fp32 columns; lane i of the warp gets TMEM lane (quadrant*32 + i).
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
-  uint32_t r[16];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
-      "%15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// 32 lanes x 64 consecutive fp32 columns in one load and one wait.
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
-  uint32_t r[64];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
-      : "r"(taddr)
-      : "memory");
-#pragma unroll
-  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
-}
-
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + __expf(-x)); }
 __device__ __forceinline__ float gelu_f(float x) {
   const float c = 0.7978845608028654f;
@@ -328,7 +232,7 @@ __device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int
 template <int TM, int BN>
 __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
-              int N, int K, int* err) {
+              int N, int K, int* err, unsigned long long wait_ns) {
   using C = Cfg<TM, BN>;
   constexpr int A_BYTES = C::A_BYTES, B_BYTES = C::B_BYTES, STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES;
   constexpr int TMEM_COLS = C::TMEM_COLS, MH = C::MH, NACC = C::NACC, EPI_WARPS = C::EPI_WARPS;
@@ -391,7 +295,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
         const int mb = tile % num_m, nb = tile / num_m;
         for (int kb = 0; kb < num_k; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, wait_ns)) {
             ok = false;
             break;
           }
@@ -406,10 +310,11 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       if (!ok) {
         atomicExch(err, 1);
         *abort_flag = 1;
-        // drain: every armed copy completes its stage's phase before the CTA exits
-        for (int s = 0; s < STAGES; ++s)
-          if (armed[s]) mbar_wait(&full[s], armed_par[s], nullptr);
       }
+      // drain: every armed copy completes its stage's phase before the CTA exits (immediate after a normal run,
+      // where the MMAs consumed them; needed when another role gave up while copies were in flight)
+      for (int s = 0; s < STAGES; ++s)
+        if (armed[s]) mbar_wait(&full[s], armed_par[s], nullptr);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -420,14 +325,14 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       uint32_t acc_phase = 0;
       bool ok = true;
       for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, wait_ns)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * ACC_COLS);
         for (int kb = 0; kb < num_k; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag)) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, wait_ns)) {
             ok = false;
             break;
           }
@@ -465,7 +370,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     for (int tile = t0; tile < num_tiles; tile += tstep) {
       const int mb = tile % num_m, nb = tile / num_m;
       // one lane waits and broadcasts, so the warp-collective tcgen05.ld below stays converged
-      int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag) : 0;
+      int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag, wait_ns) : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) {
         if (lane == 0) {
@@ -988,6 +893,9 @@ int g_bn_override = 0;  // SR_GEMM_BN: force one N-tile width (tuning sweeps)
 int g_tm_override = 0;  // SR_GEMM_TM: force the tile height (128 or 256)
 int g_pair_override = -1;  // SR_GEMM_PAIR: 1 forces the CTA-pair kernel, 0 forbids it
 int g_skinny_override = -1;  // SR_GEMM_SKINNY: 0 forbids the skinny kernel (else used for M <= 512)
+// SR_GEMM_WAIT_NS: bound of the one-SM kernel's pipeline waits (tests make it expire; the drains of copies and
+// MMAs already issued keep the 2 s bound, so an expired wait ends the kernel cleanly with the error word set)
+unsigned long long g_wait_ns = WAIT_NS;
 std::mutex g_ws_mu;
 // split-K partial workspace (floats) per (device, stream): launches on one stream run in order, so one
 // buffer per stream keeps contexts on different streams from sharing it.  sr_destroy frees the buffers
@@ -1037,7 +945,8 @@ sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs&
     max_ctas = g_num_sms;
   }
   const int tiles = ((M + TM - 1) / TM) * ((N + BN - 1) / BN);
-  launch_k(k_gemm_tc<TM, BN>, std::min(tiles, max_ctas), C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err);
+  launch_k(k_gemm_tc<TM, BN>, std::min(tiles, max_ctas), C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err,
+           g_wait_ns);
   SR_CUDA(cudaGetLastError());
   return SR_OK;
 }
@@ -1210,12 +1119,12 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     int dev;
     SR_CUDA(cudaGetDevice(&dev));
     SR_CUDA(cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev));
-    SR_CUDA(cudaMalloc(&g_err, sizeof(int)));
-    SR_CUDA(cudaMemset(g_err, 0, sizeof(int)));
+    if (!tc_error_word()) return set_err(SR_ERR_OOM, "gemm: error word allocation failed");
     if (const char* e = getenv("SR_GEMM_BN")) g_bn_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_TM")) g_tm_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_PAIR")) g_pair_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_SKINNY")) g_skinny_override = atoi(e);
+    if (const char* e = getenv("SR_GEMM_WAIT_NS")) g_wait_ns = strtoull(e, nullptr, 10);
   }
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
   CUtensorMap ta, tb;
@@ -1239,6 +1148,39 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
   if (bn == 64) return launch_bn<128, 64>(ta, tb, ep, M, N, K, st);
   if (bn == 128) return launch_bn<128, 128>(ta, tb, ep, M, N, K, st);
   return launch_bn<128, 256>(ta, tb, ep, M, N, K, st);
+}
+
+// The device error word shared by the kernels with bounded waits (allocated on first use; nullptr when
+// the allocation failed, in which case waits still end but are not reported).
+int* tc_error_word() {
+  if (!g_err) {
+    if (cudaMalloc(&g_err, sizeof(int)) != cudaSuccess) {
+      g_err = nullptr;
+      return nullptr;
+    }
+    cudaMemset(g_err, 0, sizeof(int));
+  }
+  return g_err;
+}
+
+sr_status encode_tma_2d(CUtensorMap* map, const void* base, bool bf, int rows, int cols, int box_rows) {
+  return encode_kmajor(map, base, bf, rows, cols, box_rows);
+}
+
+sr_status encode_tma_nd(CUtensorMap* map, const void* base, bool bf, int rank, const uint64_t* dims,
+                        const uint64_t* strides_bytes, const uint32_t* box) {
+  CUtensorMap tmp;
+  SR_TRY(encode_kmajor(&tmp, base, bf, 1, 64, 1));  // resolves the driver entry point once
+  cuuint64_t d[5];
+  cuuint64_t st[4];
+  cuuint32_t bx[5], es[5];
+  for (int i = 0; i < rank; ++i) d[i] = dims[i], bx[i] = box[i], es[i] = 1;
+  for (int i = 0; i + 1 < rank; ++i) st[i] = strides_bytes[i];
+  CUresult r = g_encode(map, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, (cuuint32_t)rank,
+                        const_cast<void*>(base), d, st, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return set_err(SR_ERR_INVALID_ARG, "cuTensorMapEncodeTiled (rank %d) failed (%d)", rank, (int)r);
+  return SR_OK;
 }
 
 // Device error word of the tensor-core GEMM (nonzero after a bounded wait expired).

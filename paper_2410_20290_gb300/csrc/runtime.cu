@@ -290,6 +290,9 @@ struct Work {
   char *q = nullptr, *k = nullptr, *v = nullptr, *att = nullptr, *h = nullptr;
   float* gu = nullptr;
   float* part = nullptr;
+  float* sseg = nullptr;  // streaming decode attention: segment partials and per-(row, kv head) counters
+  int* scnt = nullptr;
+  size_t c_sseg = 0, c_scnt = 0;
   int rows = 0;
 
   sr_status ensure(const Model& m, int n) {
@@ -309,12 +312,40 @@ struct Work {
     return SR_OK;
   }
   void release() {
-    void* ps[] = {x, xn, qkv, q, k, v, att, h, gu, part};
+    void* ps[] = {x, xn, qkv, q, k, v, att, h, gu, part, sseg, scnt};
     for (void* p : ps)
       if (p) cudaFree(p);
     *this = Work();
   }
 };
+
+int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+// Workspace of the streaming decode-attention kernel for b rows of Hq query heads (counters zeroed when
+// they are first allocated; every launch leaves them zero).
+sr_status stream_ws(Work& w, int b, int Hq, int pool_pages, cudaStream_t st, DecodeStreamWs* ws) {
+  const int grid = num_sms();
+  SR_TRY(grow(w.sseg, w.c_sseg, decode_stream_part_floats(grid, Hq)));
+  if (w.c_scnt < (size_t)b * 8) {
+    SR_TRY(grow(w.scnt, w.c_scnt, (size_t)b * 8));
+    SR_CUDA(cudaMemsetAsync(w.scnt, 0, w.c_scnt * sizeof(int), st));
+  }
+  ws->seg_part = w.sseg;
+  ws->seg_cnt = w.scnt;
+  ws->grid = grid;
+  ws->pool_pages = pool_pages;
+  ws->err = tc_error_word();
+  return SR_OK;
+}
 
 // Attention layout of one prefill call (packed sequences, optional shared prefix per layer).
 struct PrefillPlan {
@@ -336,6 +367,7 @@ struct PrefillPlan {
   const int* seq_cand = nullptr;     // device [n_seq]
   const int* seq_cached = nullptr;   // device [n_seq]
   int max_cached = 0;
+  int cache_pages = 0;               // pages per layer of the cache pool
 };
 // Where a prefill's per-layer K/V goes.
 struct PrefillKv {
@@ -411,6 +443,7 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
       ck.pt_stride = plan.cache_pt_stride;
       ck.seq_cand = plan.seq_cand;
       ck.seq_cached = plan.seq_cached;
+      ck.pool_pages = plan.cache_pages;
     }
     const double kvb = (double)m.kv_tok_elems() * m.esz;
     {
@@ -419,7 +452,7 @@ sr_status forward_prefill(const Model& m, Work& w, int M, const int* tok, const 
       if (m.et == SR_DT_F16)
         SR_TRY(launch_prefill_attention(m.et, w.q, kout, vout, pk, pv, plan.n_pre, plan.seq_off, plan.n_seq,
                                         plan.tile_seq, plan.tile_q0, plan.n_tiles, plan.pos0, Hq, Hkv, dh, d.window,
-                                        w.att, st, ck));
+                                        w.att, st, ck, M));
       else
         SR_TRY(launch_prefill_attention_f32((const float*)w.q, (const float*)kout, (const float*)vout,
                                             (const float*)pk, (const float*)pv, plan.n_pre, plan.seq_off, plan.n_seq,
@@ -535,7 +568,8 @@ sr_status read_ctrl(sr_ctx* c) {
   if (gerr) SR_CUDA(cudaMemcpyAsync(c->h_ctrl + C_N, gerr, sizeof(int), cudaMemcpyDeviceToHost, c->st));
   SR_CUDA(cudaStreamSynchronize(c->st));
   if (gerr && c->h_ctrl[C_N] != 0)
-    return set_err(SR_ERR_TIMEOUT, "tensor-core GEMM wait expired (code %d)", c->h_ctrl[C_N]);
+    return set_err(SR_ERR_TIMEOUT, "a bounded device wait expired (code %d: 1-3 tensor-core GEMM, 10 decode attention)",
+                   c->h_ctrl[C_N]);
   c->prof.harvest();
   if (c->h_ctrl[C_ERR] == E_POOL_EMPTY) return set_err(SR_ERR_OOM, "KV page pool exhausted");
   if (c->h_ctrl[C_ERR] == E_STATE) return set_err(SR_ERR_STATE, "no completed candidate");
@@ -659,6 +693,8 @@ sr_status prefill_prompt(sr_ctx* c, sr_batch& b) {
     SR_TRY(ctl_prompt_pages(c->free_stack, c->ctrl, b.n_sh, b.has_tail, c->pool_cap_pages - 1, c->prompt_row,
                             c->st));
   }
+  // the prompt's page ids are used by the KV writes below: stop with SR_ERR_OOM if the pool could not give them
+  SR_TRY(read_ctrl(c));
   PrefillKv gkv;
   gkv.pool = c->pool;
   gkv.pool_layer_bytes = pool_layer_bytes(c);
@@ -685,6 +721,8 @@ sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
     SR_TRY(ctl_admit(start, count, b.n_sh, b.has_tail, c->prompt_row, c->pt, b.max_pages, c->len, c->status,
                      c->live, c->rset, c->free_stack, c->ctrl, c->tail_dst, c->st));
   }
+  // the tail pages the admission popped are copied into below: stop with SR_ERR_OOM if it could not pop them
+  if (b.has_tail) SR_TRY(read_ctrl(c));
   if (b.has_tail) {
     Scope sc(pf, SR_KC_ELEMENTWISE, c->st);
     SR_TRY(launch_copy_page(g.et, c->pool, (long long)(pool_layer_bytes(c) / g.esz), g.d.n_layers,
@@ -733,6 +771,8 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host, bool sync = tr
   const int shared_pos = (m.et == SR_DT_F16 && b.n_sh > 0) ? PAGE * b.n_sh : 0;
   const int splits = decode_attention_slots(max_len, d.window, shared_pos);
   if (splits > 1) SR_TRY(grow(w.part, w.c_part, decode_attention_part_floats(n, Hq, dh, splits)));
+  DecodeStreamWs sws;
+  SR_TRY(stream_ws(w, n, Hq, c->pool_cap_pages, st, &sws));
   // algorithmic work of one decode-attention launch: the shared prompt KV once, each candidate's own KV,
   // q in and the output out
   const double kvb = 2.0 * Hkv * dh * m.esz;
@@ -759,7 +799,7 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host, bool sync = tr
     {
       Scope sc(pf, SR_KC_ATTN_DECODE, st, attn_flops, attn_bytes);
       SR_TRY(launch_decode_attention(m.et, w.q, pool_l, c->pt, b.max_pages, c->live, c->kv_len, n, Hq, Hkv, dh,
-                                     d.window, w.att, w.part, splits, st, shared_pos, max_len));
+                                     d.window, w.att, w.part, splits, st, shared_pos, max_len, nullptr, &sws));
     }
     SR_TRY(linear(m, w.att, lw.wo, w.x, n, D, Hq * dh, EPI_ADD_F32, st, pf, SR_KC_GEMM_DECODE));
     {
@@ -976,6 +1016,7 @@ sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std
       plan.seq_cand = did;
       plan.seq_cached = dc;
       plan.max_cached = max_cached;
+      plan.cache_pages = rc.pages;
       if (store) {
         kv.pool = c->rm_pool;
         kv.pool_layer_bytes = cache_layer;
@@ -1521,9 +1562,22 @@ sr_status sr_k_decode_attention(int dtype, const void* q, const void* pool, cons
   float* part = nullptr;
   if (splits > 1) SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&part),
                                           decode_attention_part_floats(b, n_heads, head_dim, splits) * sizeof(float), st));
+  // the streaming kernel's workspace.  The pool's size is not an argument here, so its tensor map spans the
+  // largest page count a 2D map can address; the kernel reads only the pages the page table names, as the
+  // per-row kernels do.
+  DecodeStreamWs ws;
+  ws.grid = num_sms();
+  ws.err = tc_error_word();
+  SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&ws.seg_part),
+                          decode_stream_part_floats(ws.grid, n_heads) * sizeof(float), st));
+  SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&ws.seg_cnt), (size_t)std::max(b, 1) * 8 * sizeof(int), st));
+  SR_CUDA(cudaMemsetAsync(ws.seg_cnt, 0, (size_t)std::max(b, 1) * 8 * sizeof(int), st));
+  ws.pool_pages = (int)(((1u << 31) - 1) / (2u * 8u * PAGE));
   sr_status s = launch_decode_attention(dtype, q, pool, page_table, pt_stride, orig_ids, lens, b, n_heads, n_kv_heads,
-                                        head_dim, window, out, part, splits, st, shared_pos, mx);
+                                        head_dim, window, out, part, splits, st, shared_pos, mx, nullptr, &ws);
   if (part) cudaFreeAsync(part, st);
+  cudaFreeAsync(ws.seg_part, st);
+  cudaFreeAsync(ws.seg_cnt, st);
   return s;
 }
 
@@ -1546,7 +1600,7 @@ sr_status sr_k_prefill_attention(int dtype, const void* q, const void* k, const 
   hcat.insert(hcat.end(), tq.begin(), tq.end());
   SR_CUDA(cudaMemcpyAsync(d, hcat.data(), 2 * nt * sizeof(int), cudaMemcpyHostToDevice, st));
   sr_status s = launch_prefill_attention(dtype, q, k, v, k_pre, v_pre, n_pre, seq_off, n_seq, d, d + nt, nt, pos0,
-                                         n_heads, n_kv_heads, head_dim, window, out, st);
+                                         n_heads, n_kv_heads, head_dim, window, out, st, CachedKeys(), off[n_seq]);
   cudaStreamSynchronize(st);  // the host copy of the tile list must outlive the upload
   cudaFreeAsync(d, st);
   return s;

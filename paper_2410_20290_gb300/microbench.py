@@ -4,6 +4,7 @@
   python -m paper_2410_20290_gb300.microbench decode_attn b Hq Hkv dh len [shared_positions]
   python -m paper_2410_20290_gb300.microbench prefill_attn n_seq tau n_pre Hq Hkv dh
   python -m paper_2410_20290_gb300.microbench sample b V
+  python -m paper_2410_20290_gb300.microbench decode_gemms M
 
 Prints one JSON line with the mean launch time and the achieved rate (TFLOP/s or GB/s) of the
 algorithmic work.  Operands are sized by the shape given; choose shapes larger than the 129 MB L2
@@ -93,9 +94,25 @@ def sample(b, V, iters=20):
     return dict(kernel="sample", b=b, V=V, ms=ms, gbs=b * V * 4 / ms / 1e6)
 
 
+def decode_gemms(M, iters=5):
+    """The five GEMMs of one decode step of the Llama-3-8B-shaped generator at M live rows (QKV, O + residual,
+    gate/up + SwiGLU, down + residual, LM head), each launched `iters` times; per shape the mean time and the
+    algorithmic bytes of one launch (operands read once, result written once; + the residual read)."""
+    shapes = (("qkv", 6144, 4096, 0), ("o", 4096, 4096, 1), ("gate_up", 28672, 4096, 3), ("down", 4096, 14336, 1),
+              ("lm_head", 128256, 4096, 0))
+    out = []
+    for name, N, K, epi in shapes:
+        r = gemm(M, N, K, epi, iters)
+        out_b = {0: 4 * M * N, 1: 8 * M * N, 3: M * N}[epi]
+        r.update(name=name, alg_bytes=2 * (M * K + N * K) + out_b)
+        out.append(r)
+    return dict(kernel="decode_gemms", M=M, shapes=out)
+
+
 def main(argv):
     kind, nums = argv[0], [int(x) for x in argv[1:]]
-    fn = {"gemm": gemm, "decode_attn": decode_attn, "prefill_attn": prefill_attn, "sample": sample}[kind]
+    fn = {"gemm": gemm, "decode_attn": decode_attn, "prefill_attn": prefill_attn, "sample": sample,
+          "decode_gemms": decode_gemms}[kind]
     print(json.dumps(fn(*nums)), flush=True)
 
 

@@ -174,6 +174,13 @@ def _round16(x, dt=si.DT_F16):
     # suffixes of at most 8 pages run one warp per (kv head, slot); 2 kv heads leave two warps idle
     (si.DT_F16, 16, 2, 128, 0, [289, 300, 310, 390], 288),
     (si.DT_F16, 32, 8, 128, 0, [257, 258, 270, 300, 384] * 40, 256),
+    # head_dim 128 with 8 kv heads runs the streaming kernel: fewer pages than SMs, group sizes 1, 2 and 8,
+    # and a few hundred rows whose pages the per-SM shares cut at many places
+    (si.DT_F16, 8, 8, 128, 0, [5, 17, 40], 0),
+    (si.DT_F16, 16, 8, 128, 0, [100, 700, 1500], 0),
+    (si.DT_F16, 64, 8, 128, 0, [64, 513, 1025], 0),
+    (si.DT_F16, 8, 8, 128, 0, [290 + (13 * i) % 200 for i in range(300)], 288),
+    (si.DT_BF16, 32, 8, 128, 64, [300 + (3 * i) % 400 for i in range(200)], 128),
 ])
 def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens, shared):
     rng = np.random.default_rng(dh + len(lens))
@@ -210,6 +217,13 @@ def test_decode_attention(sr, dt, Hq, Hkv, dh, window, lens, shared):
     (si.DT_F16, 4, 2, 128, 0, [300], 0),
     (si.DT_F16, 8, 4, 64, 40, [90, 33], 50),
     (si.DT_BF16, 32, 8, 128, 288, [1, 64, 65, 200, 7], 0),
+    # head_dim 128 with 8 kv heads runs the tcgen05 kernel: group sizes 1, 2 and 8, a window, a 512-position
+    # prefix, and own rows over several 128-key blocks
+    (si.DT_F16, 8, 8, 128, 100, [70, 1, 128], 0),
+    (si.DT_F16, 16, 8, 128, 0, [300, 17], 0),
+    (si.DT_F16, 64, 8, 128, 40, [90, 33], 50),
+    (si.DT_F16, 32, 8, 128, 512, [600, 5, 129], 0),
+    (si.DT_BF16, 32, 8, 128, 130, [257, 31], 200),
 ])
 def test_prefill_attention(sr, dt, Hq, Hkv, dh, n_pre, taus, window):
     rng = np.random.default_rng(dh + n_pre)

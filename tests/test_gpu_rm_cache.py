@@ -138,3 +138,14 @@ def test_gqa_head_dim_256_reward_model_with_cache(sr):
         _component_run(sr, w, ctx, gw, rw, w.prompt(0), 2, (9, 18), 0.5)
     finally:
         sr.sr_destroy(ctx)
+
+
+def test_llama_width_reward_model_with_cache(sr):
+    """8B widths (head_dim 128, 8 kv heads: the tensor-core prefill kernel reads the cached pages), 2 layers:
+    rounds at 7 and 15 tokens and the final scoring with the cache, each against the oracle's full rescoring."""
+    w = si.shrink(si.WORKLOADS["llama8b_n256"], 2, N=8, max_new=24, taus=(), prompt_len=40, pool_bytes=0)
+    ctx, gw, rw = _ctx(sr, w, 2)
+    try:
+        _component_run(sr, w, ctx, gw, rw, w.prompt(3), 5, (7, 15), 0.5)
+    finally:
+        sr.sr_destroy(ctx)
