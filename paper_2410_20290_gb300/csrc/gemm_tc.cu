@@ -175,65 +175,118 @@ __device__ __forceinline__ void umma_pair_commit_mc(uint64_t* bar, uint16_t mask
 // Epilogue of one accumulator row segment: this thread's row of BNC fp32 columns at TMEM address
 // `tbase`, converted / activated / added and stored at (row, col0 ..).  Rows >= M and columns >= N are
 // skipped (they hold the zero-filled tails of the TMA tiles).
-template <int BNC>
-__device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int row, int col0, int M, int N) {
+// Epilogue of 64 accumulator values v (columns col .. col + 63 of `row`): conversion / residual add / gated or
+// GELU activation and the store.  Rows >= M and columns >= N are skipped (the zero-filled tails of the tiles).
+__device__ __forceinline__ void epi_chunk(const EpiArgs& ep, float* v, int row, int col, int M, int N) {
   if (ep.kind == EPI_SWIGLU || ep.kind == EPI_GEGLU) {
-#pragma unroll 1
-    for (int c = 0; c < BNC; c += 64) {
-      // gate / up rows interleaved in blocks of 16: columns c..c+15 gate, c+16..c+31 up, c+32.. the next pair
-      float v[64];
-      tmem_ld64(tbase + c, v);
-      if (row < M && col0 + c < N) {
-        float g[32];
+    // gate / up rows interleaved in blocks of 16: columns col..col+15 gate, col+16..col+31 up, then the next pair
+    if (row < M && col < N) {
+      float g[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int gi = (j < 16) ? j : j + 16;
-          g[j] = (ep.kind == EPI_SWIGLU ? silu_f(v[gi]) : gelu_f(v[gi])) * v[gi + 16];
-        }
-        uint16_t* dst = reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + (col0 + c) / 2;
-        store16x32(dst, g, ep.bf != 0);
+      for (int j = 0; j < 32; ++j) {
+        const int gi = (j < 16) ? j : j + 16;
+        g[j] = (ep.kind == EPI_SWIGLU ? silu_f(v[gi]) : gelu_f(v[gi])) * v[gi + 16];
       }
+      uint16_t* dst = reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col / 2;
+      store16x32(dst, g, ep.bf != 0);
     }
-  } else {
-#pragma unroll 1
-    for (int c = 0; c < BNC; c += 64) {
-      float v[64];
-      tmem_ld64(tbase + c, v);
+    return;
+  }
 #pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        float* w = v + 32 * hh;
-        const int cc = c + 32 * hh;
-        if (row < M && col0 + cc < N) {
-          if (ep.kind == EPI_F32 || ep.kind == EPI_ADD_F32) {
-            float4* dst =
-                reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)row * ep.ldo + col0 + cc);
+  for (int hh = 0; hh < 2; ++hh) {
+    float* w = v + 32 * hh;
+    const int cc = col + 32 * hh;
+    if (row < M && cc < N) {
+      if (ep.kind == EPI_F32 || ep.kind == EPI_ADD_F32) {
+        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) + (size_t)row * ep.ldo + cc);
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              float4 o = make_float4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-              if (ep.kind == EPI_ADD_F32) {
-                const float4 r = dst[q];
-                o.x += r.x, o.y += r.y, o.z += r.z, o.w += r.w;
-              }
-              dst[q] = o;
-            }
-          } else {
-            if (ep.kind == EPI_GELU) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j) w[j] = gelu_f(w[j]);
-            }
-            store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + col0 + cc, w, ep.bf != 0);
+        for (int q = 0; q < 8; ++q) {
+          float4 o = make_float4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+          if (ep.kind == EPI_ADD_F32) {
+            const float4 r = dst[q];
+            o.x += r.x, o.y += r.y, o.z += r.z, o.w += r.w;
           }
+          dst[q] = o;
         }
+      } else {
+        if (ep.kind == EPI_GELU) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) w[j] = gelu_f(w[j]);
+        }
+        store16x32(reinterpret_cast<uint16_t*>(ep.out) + (size_t)row * ep.ldo + cc, w, ep.bf != 0);
       }
     }
   }
 }
 
+// Epilogue of one accumulator row segment: this thread's row of BNC fp32 columns at TMEM address `tbase`,
+// 64 columns per load and wait.
+template <int BNC>
+__device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int row, int col0, int M, int N) {
+#pragma unroll 1
+  for (int c = 0; c < BNC; c += 64) {
+    float v[64];
+    tmem_ld64(tbase + c, v);
+    epi_chunk(ep, v, row, col0 + c, M, N);
+  }
+}
+
+// Tile t -> (M tile, N tile): groups of up to RASTER_M consecutive M tiles, M fastest within a group and the
+// group's N tiles in order, so the CTAs resident at one time share a band of A rows that stays in L2 while W
+// streams past (a single group -- every shape up to RASTER_M M tiles -- is plain M-fastest order).
+constexpr int RASTER_M = 16;
+__device__ __forceinline__ void tile_mn(int t, int num_m, int num_n, int& mb, int& nb) {
+  const int per_group = RASTER_M * num_n;
+  const int g = t / per_group, r = t - g * per_group;
+  const int m0 = g * RASTER_M, gm = min(RASTER_M, num_m - m0);
+  mb = m0 + r % gm;
+  nb = r / gm;
+}
+
+// Stream-K: the num_tiles x num_k k-block units of a launch, tile by tile, are cut into gridDim.x contiguous
+// shares of (almost) equal size; a CTA's share is a run of segments (tile, k-blocks kb0..kb1).  A segment that
+// is not a whole tile writes its fp32 accumulator rows to one of the CTA's two partial slots (the share's first
+// or last segment) and each epilogue warp counts its 32 rows on the tile's counter for its lane quadrant; the
+// last of a tile's segments for those rows sums the slots in CTA order -- k order, so the result does not
+// depend on which CTA finishes last -- applies the epilogue and resets the counter.  No warp waits on another.
+struct SkArgs {
+  float* part = nullptr;  // [gridDim.x][2] slots of [BN / 4][TM] float4
+  int* cnt = nullptr;     // [num_tiles][4] (tile, TMEM lane quadrant), zero between launches
+  int on = 0;
+};
+struct Seg {
+  int tile, kb0, kb1;
+};
+__device__ __forceinline__ long long sk_share(long long total, int c, int C) { return total * c / C; }
+__device__ __forceinline__ int sk_cta_of(long long u, long long total, int C) {
+  int i = (int)(u * C / total);
+  while (i + 1 < C && sk_share(total, i + 1, C) <= u) ++i;
+  while (i > 0 && sk_share(total, i, C) > u) --i;
+  return i;
+}
+// The i-th segment of this CTA (false past the last): whole tiles t0 + i tstep without stream-K.
+__device__ __forceinline__ bool sk_segment(bool on, int i, int num_tiles, int num_k, long long u0, long long u1,
+                                           int t0, int tstep, long long& cursor, Seg& sg) {
+  if (!on) {
+    const int t = t0 + i * tstep;
+    if (t >= num_tiles) return false;
+    sg = Seg{t, 0, num_k};
+    return true;
+  }
+  if (cursor >= u1) return false;
+  const int t = (int)(cursor / num_k), kb0 = (int)(cursor % num_k);
+  const int kb1 = (int)min((long long)num_k, kb0 + (u1 - cursor));
+  sg = Seg{t, kb0, kb1};
+  cursor += kb1 - kb0;
+  return true;
+}
+
 template <int TM, int BN>
 __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
-              int N, int K, int* err, unsigned long long wait_ns) {
+              int N, int K, int* err, unsigned long long wait_ns, SkArgs sk) {
   using C = Cfg<TM, BN>;
+  static_assert(TM == 128 || TM == 256, "tile height");
   constexpr int A_BYTES = C::A_BYTES, B_BYTES = C::B_BYTES, STAGE_BYTES = C::STAGE_BYTES, STAGES = C::STAGES;
   constexpr int TMEM_COLS = C::TMEM_COLS, MH = C::MH, NACC = C::NACC, EPI_WARPS = C::EPI_WARPS;
   constexpr int ACC_COLS = MH * BN;  // TMEM columns of one accumulator buffer
@@ -253,9 +306,13 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
   const uint32_t idesc = idesc_for(ep.bf != 0, BN);
   const int num_m = (M + TM - 1) / TM, num_n = (N + BN - 1) / BN;
   const int num_k = (K + BK - 1) / BK;
-  // tiles of this CTA: index t over (M tile, N tile), M fastest
+  // tiles of this CTA: index t over (M tile, N tile), M fastest; with stream-K (TM = 128) a share of k-block units
   const int num_tiles = num_m * num_n;
   const int t0 = blockIdx.x, tstep = gridDim.x;
+  const bool skon = TM == 128 && sk.on;
+  const long long sk_total = (long long)num_tiles * num_k;
+  const long long u0 = skon ? sk_share(sk_total, blockIdx.x, gridDim.x) : 0;
+  const long long u1 = skon ? sk_share(sk_total, blockIdx.x + 1, gridDim.x) : 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -292,9 +349,12 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       uint32_t armed_par[STAGES];
       for (int s = 0; s < STAGES; ++s) armed[s] = 0, armed_par[s] = 0;
       bool ok = true;
-      for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
-        const int mb = tile % num_m, nb = tile / num_m;
-        for (int kb = 0; kb < num_k; ++kb) {
+      long long cur = u0;
+      Seg sg;
+      for (int i = 0; ok && sk_segment(skon, i, num_tiles, num_k, u0, u1, t0, tstep, cur, sg); ++i) {
+        int mb, nb;
+        tile_mn(sg.tile, num_m, num_n, mb, nb);
+        for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, wait_ns)) {
             ok = false;
             break;
@@ -324,14 +384,16 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
+      long long cur = u0;
+      Seg sg;
+      for (int i = 0; ok && sk_segment(skon, i, num_tiles, num_k, u0, u1, t0, tstep, cur, sg); ++i) {
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, wait_ns)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * ACC_COLS);
-        for (int kb = 0; kb < num_k; ++kb) {
+        for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, wait_ns)) {
             ok = false;
             break;
@@ -344,7 +406,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes per K=16 step inside the swizzle atom
               umma(d_tmem + (uint32_t)(h * BN), a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc,
-                   (kb | kk) != 0);
+                   (kb != sg.kb0 || kk != 0) ? 1u : 0u);
           }
           umma_commit(&empty[stage]);
           if (++stage == STAGES) stage = 0, phase ^= 1u;
@@ -367,8 +429,12 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     const int quad = warp & 3, half = (warp - 2) / 4;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = t0; tile < num_tiles; tile += tstep) {
-      const int mb = tile % num_m, nb = tile / num_m;
+    long long cur = u0;
+    Seg sg;
+    for (int i = 0; sk_segment(skon, i, num_tiles, num_k, u0, u1, t0, tstep, cur, sg); ++i) {
+      const int tile = sg.tile;
+      int mb, nb;
+      tile_mn(tile, num_m, num_n, mb, nb);
       // one lane waits and broadcasts, so the warp-collective tcgen05.ld below stays converged
       int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag, wait_ns) : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -382,11 +448,60 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       tc_fence_after();
       const int row = mb * TM + half * BM + quad * 32 + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * ACC_COLS + half * BN);
-      epi_store<BN>(ep, tbase, row, nb * BN, M, N);
+      if (sg.kb0 == 0 && sg.kb1 == num_k) {
+        epi_store<BN>(ep, tbase, row, nb * BN, M, N);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        if (++acc == NACC) acc = 0, acc_phase ^= 1u;
+        continue;
+      }
+      // ---- a part of the tile: fp32 rows to this CTA's slot, then the tile's counter ----
+      const long long ts = (long long)tile * num_k;
+      const int which = ts >= u0 ? 1 : 0;  // the tile began inside the share: the share's last segment
+      // slot layout [column group of 4][row]: a warp's float4 accesses cover 512 contiguous bytes
+      const int r = quad * 32 + lane;       // row within the tile (TM = 128)
+      float4* slot = reinterpret_cast<float4*>(sk.part) + ((size_t)blockIdx.x * 2 + which) * (TM * BN / 4) + r;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 64) {
+        float v[64];
+        tmem_ld64(tbase + c, v);
+#pragma unroll
+        for (int q = 0; q < 16; ++q)
+          __stcg(slot + (size_t)(c / 4 + q) * TM, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+      }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (lane == 0) mbar_arrive(&tempty[acc]);  // the accumulator is free for the next segment
       if (++acc == NACC) acc = 0, acc_phase ^= 1u;
+      // each epilogue warp counts its own 32 rows (one counter per tile and lane quadrant), so no warp waits on
+      // another; the last of the tile's segments for these rows merges them
+      __threadfence();
+      __syncwarp();
+      const int c0 = sk_cta_of(ts, sk_total, gridDim.x), c1 = sk_cta_of(ts + num_k - 1, sk_total, gridDim.x);
+      int last = 0;
+      if (lane == 0) last = atomicAdd(&sk.cnt[(size_t)tile * 4 + quad], 1) == c1 - c0;
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (!last) continue;
+      __threadfence();
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 64) {
+        float v[64];
+#pragma unroll
+        for (int e = 0; e < 64; ++e) v[e] = 0.f;
+        for (int cc = c0; cc <= c1; ++cc) {  // k order
+          // the writer's slot rule: slot 1 where the tile began inside the writer's share (only c0's can)
+          const int wc = sk_share(sk_total, cc, gridDim.x) <= ts ? 1 : 0;
+          const float4* src = reinterpret_cast<const float4*>(sk.part) + ((size_t)cc * 2 + wc) * (TM * BN / 4) + r;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const float4 p = __ldcg(src + (size_t)(c / 4 + q) * TM);  // L2: written by other SMs
+            v[4 * q] += p.x, v[4 * q + 1] += p.y, v[4 * q + 2] += p.z, v[4 * q + 3] += p.w;
+          }
+        }
+        epi_chunk(ep, v, row, nb * BN + c, M, N);
+      }
+      if (lane == 0) sk.cnt[(size_t)tile * 4 + quad] = 0;
     }
   }
   tc_fence_before();
@@ -491,7 +606,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       for (int s = 0; s < STAGES; ++s) armed[s] = 0, armed_par[s] = 0;
       bool ok = true;
       for (int tile = t0; tile < num_tiles && ok; tile += tstep) {
-        const int mb = tile % num_m, nb = tile / num_m;
+        int mb, nb;
+      tile_mn(tile, num_m, num_n, mb, nb);
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) {
             ok = false;
@@ -567,7 +683,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = t0; tile < num_tiles; tile += tstep) {
-      const int mb = tile % num_m, nb = tile / num_m;
+      int mb, nb;
+      tile_mn(tile, num_m, num_n, mb, nb);
       int ok = (lane == 0) ? (int)mbar_wait(&tfull[acc], acc_phase, abort_flag) : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) {
@@ -896,6 +1013,10 @@ int g_skinny_override = -1;  // SR_GEMM_SKINNY: 0 forbids the skinny kernel (els
 // SR_GEMM_WAIT_NS: bound of the one-SM kernel's pipeline waits (tests make it expire; the drains of copies and
 // MMAs already issued keep the 2 s bound, so an expired wait ends the kernel cleanly with the error word set)
 unsigned long long g_wait_ns = WAIT_NS;
+// SR_GEMM_STREAMK=1: stream-K shares of k-blocks on 128 x 256 tiles for every shape with a k-block per SM.  Off
+// by default: on GB300 it measured slower than the launcher's tile choices on every decode shape (the merge of
+// a tile's partial sums by its last contributor costs more than the idle SMs of the last wave).
+int g_sk_override = 0;
 std::mutex g_ws_mu;
 // split-K partial workspace (floats) per (device, stream): launches on one stream run in order, so one
 // buffer per stream keeps contexts on different streams from sharing it.  sr_destroy frees the buffers
@@ -935,9 +1056,45 @@ bool pick_tall(int M, int N, int K) {
   return t_tall < t_small;
 }
 
+// Stream-K workspace per (device, stream): partial slots and the per-(tile, quadrant) counters, zeroed when
+// allocated (every launch leaves them zero).
+struct SkWs {
+  float* part = nullptr;
+  size_t part_cap = 0;
+  int* cnt = nullptr;
+  size_t cnt_cap = 0;
+};
+std::map<std::pair<int, cudaStream_t>, SkWs> g_skws;
+
+sr_status sk_workspace(size_t part_floats, size_t cnt_ints, cudaStream_t st, SkArgs* sk) {
+  int dev;
+  SR_CUDA(cudaGetDevice(&dev));
+  std::lock_guard<std::mutex> lk(g_ws_mu);
+  SkWs& w = g_skws[std::make_pair(dev, st)];
+  if (w.part_cap < part_floats) {
+    if (w.part) SR_CUDA(cudaFree(w.part));
+    w.part = nullptr;
+    w.part_cap = 0;
+    SR_CUDA(cudaMalloc(&w.part, part_floats * sizeof(float)));
+    w.part_cap = part_floats;
+  }
+  if (w.cnt_cap < cnt_ints) {
+    if (w.cnt) SR_CUDA(cudaFree(w.cnt));
+    w.cnt = nullptr;
+    w.cnt_cap = 0;
+    SR_CUDA(cudaMalloc(&w.cnt, cnt_ints * sizeof(int)));
+    SR_CUDA(cudaMemsetAsync(w.cnt, 0, cnt_ints * sizeof(int), st));
+    w.cnt_cap = cnt_ints;
+  }
+  sk->part = w.part;
+  sk->cnt = w.cnt;
+  sk->on = 1;
+  return SR_OK;
+}
+
 template <int TM, int BN>
 sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
-                    cudaStream_t st) {
+                    cudaStream_t st, bool streamk = false) {
   using C = Cfg<TM, BN>;
   static int max_ctas = 0;
   if (!max_ctas) {
@@ -945,8 +1102,14 @@ sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs&
     max_ctas = g_num_sms;
   }
   const int tiles = ((M + TM - 1) / TM) * ((N + BN - 1) / BN);
-  launch_k(k_gemm_tc<TM, BN>, std::min(tiles, max_ctas), C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err,
-           g_wait_ns);
+  SkArgs sk;
+  int grid = std::min(tiles, max_ctas);
+  // stream-K needs a unit for every CTA (an empty share would leave a split tile's count short)
+  if (streamk && TM == 128 && (long long)tiles * ((K + BK - 1) / BK) >= max_ctas) {
+    grid = max_ctas;
+    SR_TRY(sk_workspace((size_t)grid * 2 * TM * BN, (size_t)tiles * 4, st, &sk));
+  }
+  launch_k(k_gemm_tc<TM, BN>, grid, C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err, g_wait_ns, sk);
   SR_CUDA(cudaGetLastError());
   return SR_OK;
 }
@@ -1125,11 +1288,17 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     if (const char* e = getenv("SR_GEMM_PAIR")) g_pair_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_SKINNY")) g_skinny_override = atoi(e);
     if (const char* e = getenv("SR_GEMM_WAIT_NS")) g_wait_ns = strtoull(e, nullptr, 10);
+    if (const char* e = getenv("SR_GEMM_STREAMK")) g_sk_override = atoi(e);
   }
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
   CUtensorMap ta, tb;
   EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
   const bool forced = g_pair_override == 1 || g_bn_override != 0 || g_tm_override != 0;
+  if (g_sk_override == 1) {
+    SR_TRY(encode_kmajor(&ta, A, bf, M, K, BM));
+    SR_TRY(encode_kmajor(&tb, W, bf, N, K, 256));
+    return launch_bn<128, 256>(ta, tb, ep, M, N, K, st, true);
+  }
   if (M <= 512 && g_skinny_override != 0 && (g_skinny_override == 1 || (!forced && pick_skinny(M, N, K))))
     return launch_skinny(A, W, bf, ep, M, N, K, st);
   if (g_pair_override == 1 ||
@@ -1193,9 +1362,16 @@ void gemm_release_workspace(cudaStream_t st) {
   if (cudaGetDevice(&dev) != cudaSuccess) return;
   std::lock_guard<std::mutex> lk(g_ws_mu);
   auto it = g_ws.find(std::make_pair(dev, st));
-  if (it == g_ws.end()) return;
-  if (it->second.first) cudaFree(it->second.first);
-  g_ws.erase(it);
+  if (it != g_ws.end()) {
+    if (it->second.first) cudaFree(it->second.first);
+    g_ws.erase(it);
+  }
+  auto is = g_skws.find(std::make_pair(dev, st));
+  if (is != g_skws.end()) {
+    if (is->second.part) cudaFree(is->second.part);
+    if (is->second.cnt) cudaFree(is->second.cnt);
+    g_skws.erase(is);
+  }
 }
 
 }  // namespace sr

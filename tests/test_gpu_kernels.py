@@ -103,7 +103,11 @@ T16 = {si.DT_BF16: torch.bfloat16, si.DT_F16: torch.float16}
 # 256: e.g. 1024 x 4096) and ragged M, N and K tails
 @pytest.mark.parametrize("M,N,K", [(1, 256, 64), (7, 512, 128), (130, 2304, 768), (300, 288, 1000), (257, 96, 520),
                                    (1024, 4096, 4096), (1, 32000, 768), (2048, 512, 64), (1024, 6144, 520),
-                                   (308, 28672, 256), (308, 6144, 512)])
+                                   (308, 28672, 256), (308, 6144, 512),
+                                   # with SR_GEMM_STREAMK=1: shares cut tiles mid-k (48 tiles x 32 k-blocks)
+                                   (300, 4096, 2000),
+                                   # more M tiles than one raster group (16 M tiles), ragged last group
+                                   (4500, 1024, 256)])
 def test_gemm_tc_fp32_out(sr, dt, M, N, K):
     g = torch.Generator().manual_seed(M * 7 + N + K)
     A = torch.randn(M, K, generator=g).to(T16[dt])
@@ -122,7 +126,7 @@ def test_gemm_tc_fp32_out(sr, dt, M, N, K):
 @pytest.mark.parametrize("dt", [si.DT_F16, si.DT_BF16])
 @pytest.mark.parametrize("epi", [2, 3, 4, 5])
 @pytest.mark.parametrize("M,N,K", [(5, 256, 64), (200, 1024, 512), (129, 512, 4096), (308, 6144, 512),
-                                   (1024, 4096, 64)])
+                                   (1024, 4096, 64), (308, 2048, 4096), (4500, 1024, 256)])
 def test_gemm_tc_epilogues(sr, dt, epi, M, N, K):
     g = torch.Generator().manual_seed(epi * 1000 + M)
     A = (torch.randn(M, K, generator=g) / np.sqrt(K)).to(T16[dt])
@@ -140,6 +144,24 @@ def test_gemm_tc_epilogues(sr, dt, epi, M, N, K):
     sr.sr_k_gemm(dt, A.cuda(), W.cuda(), C, M, N, K, epi)
     tol = 1.6e-2 if dt == si.DT_BF16 else 2e-3
     torch.testing.assert_close(C.float().cpu(), ref.to(T16[dt]).float(), rtol=tol, atol=1e-3)
+
+
+@pytest.mark.parametrize("M,N,K,epi", [(300, 4096, 2000, 0), (308, 28672, 4096, 3), (1024, 6144, 4096, 0),
+                                       (308, 4096, 14336, 1)])
+def test_gemm_tc_repeatable(sr, M, N, K, epi):
+    """Decode shapes, three calls: the same bits every time.  Split-K partials (the skinny kernel) and stream-K
+    shares (SR_GEMM_STREAMK=1) are summed in k order, not in the order the CTAs finish."""
+    g = torch.Generator().manual_seed(M + N + K)
+    A = (torch.randn(M, K, generator=g) / np.sqrt(K)).half().cuda()
+    W = torch.randn(N, K, generator=g).half().cuda()
+    shape = (M, N // 2) if epi == 3 else (M, N)
+    base = torch.randn(*shape, generator=g).cuda()
+    outs = []
+    for _ in range(3):
+        C = base.clone() if epi == 1 else torch.zeros(*shape, device="cuda", dtype=torch.float16 if epi == 3 else torch.float32)
+        sr.sr_k_gemm(si.DT_F16, A, W, C, M, N, K, epi)
+        outs.append(C.cpu())
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 64, 16), (33, 200, 77), (128, 512, 128)])
