@@ -34,6 +34,12 @@ import sr_inputs as si
 METRIC = "Best-of-N wall time & generated tokens/s at 8B, N=1024; HBM roofline %"
 UNIT = "generated tokens/s"
 KC = ("gemm_decode", "gemm_score", "gemm_prompt", "attn_decode", "attn_prefill", "sample", "elementwise", "control")
+# DRAM bytes (read + write) per decode-GEMM launch: one ncu pass of dram__bytes_read.sum + dram__bytes_write.sum over
+# the five decode GEMM shapes (QKV, O, gate/up, down, LM head) at 1024 and at 308 rows (the microbench's decode_gemms
+# mode), weighted by a step's launches (32 layers x 4 + 1) and by the headline run's 443 steps at 1024 rows and 580
+# at 308.  Algorithmic bytes of the same mix: 145.2 MB per launch.  Valid for the GEMM kernels as captured.
+GEMM_DECODE_TRAFFIC = {"bytes_per_launch": 140.9e6, "algorithmic_bytes_per_launch": 145.2e6,
+                       "source": "ncu dram__bytes_read.sum + dram__bytes_write.sum, decode GEMM shapes at 1024 / 308 rows"}
 
 
 def load_peaks():
@@ -442,8 +448,11 @@ def main():
         roof = None
     elif dom.startswith("gemm") or dom == "attn_prefill":
         achieved = dv["timed_flops"] / (dv["ms"] / 1e3) / 1e12
+        tr = GEMM_DECODE_TRAFFIC if (dom == "gemm_decode" and w.name == "llama8b_n1024" and args.max_new is None
+                                     and args.pool_gb is None) else None
         roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": tf_sus, "unit": "TFLOP/s",
-                "frac": round(achieved / tf_sus, 4), "traffic": None, "kernel": dom,
+                "frac": round(achieved / tf_sus, 4), "traffic": tr["bytes_per_launch"] if tr else None,
+                "traffic_note": tr, "kernel": dom,
                 "note": f"bf16 dense sustained peak ({src}); achieved = 2MNK per launch / CUDA-event launch time, "
                         f"over the {dv['timed']} launches timed (one in {args.prof_period} of each class)"}
     else:

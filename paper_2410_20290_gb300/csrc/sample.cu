@@ -11,7 +11,9 @@
 // so its bits are fixed by the method, not by the compiler.
 //
 // One block per row; each thread handles groups of 4 consecutive vocabulary ids (one Philox
-// call per group); block argmax with ties to the lowest id; NaN logits count as -inf.
+// call per group); block argmax with ties to the lowest id; NaN logits count as -inf.  The two
+// logarithms are taken only for ids that can still beat the thread's running maximum (an exact
+// test on the uniform, see k_sample), which after the first few ids of a thread is a small fraction.
 //
 // With `lp_sum` set, the same pass also takes ln sum_v exp(logit_v) of the raw logits (online
 // max / rescaled sum) and adds ln p(token) = logit_token - that to lp_sum[candidate id]: the running
@@ -115,7 +117,16 @@ __global__ void __launch_bounds__(THREADS) k_sample(const float* __restrict__ lo
       }
       if (v == eos_id) a = __fadd_rn(a, eos_bias);
       if (a != a) a = -__int_as_float(0x7f800000);
-      const float z = __fadd_rn(__fmul_rn(a, inv_t), gumbel_of(words[j]));
+      const float ap = __fmul_rn(a, inv_t);
+      // Exact skip of ids that cannot win.  g(u) = -ln(-ln u) reaches best - ap only if -ln u <= exp(ap - best),
+      // and -ln u >= 1 - u, so 1 - u > exp(ap - best + margin) proves g(u) < best - ap - margin.  The margin
+      // (1e-4 + 5 ulp of best) exceeds the error of the two series logarithms (< 1e-5 for |g| <= 17, checked
+      // over all 2^23 uniforms) plus the roundings of ap - best and of z, so a skipped id's z is strictly below
+      // this thread's best and below the row's maximum; 1 - u is exact in float32 and the 1.001 factor covers
+      // __expf's error.
+      const float one_minus_u = __fmul_rn((float)(0x7FFFFFu - (words[j] >> 9)) + 0.5f, 0x1p-23f);
+      if (one_minus_u > __expf(ap - best + (1e-4f + fabsf(best) * 6e-7f)) * 1.001f) continue;
+      const float z = __fadd_rn(ap, gumbel_of(words[j]));
       if (z > best) best = z, best_v = v;  // v increases per thread, so ">" keeps the lowest id
     }
   }

@@ -50,6 +50,33 @@ def test_sample_bit_exact(sr, V, T, bias, eos):
     assert out.cpu().numpy().tolist() == want
 
 
+@pytest.mark.parametrize("kind", ["wide", "ties", "large", "sharp"])
+def test_sample_skip_test_keeps_decisions(sr, kind):
+    """The kernel takes the logarithms only for ids that can still win (an exact bound on the uniform); the
+    decisions must equal the oracle's full Gumbel-max on spreads where most ids are skipped (wide), on exact ties
+    of the top logits (ties: lowest id wins), at large magnitudes (the margin's ulp term) and on a peaked row."""
+    rng = np.random.default_rng({"wide": 1, "ties": 2, "large": 3, "sharp": 4}[kind])
+    b, V = 48, 128256
+    if kind == "wide":
+        logits = rng.standard_normal((b, V)) * 8.0
+    elif kind == "ties":
+        logits = np.round(rng.standard_normal((b, V)) * 2.0)          # many equal values, top ones tied
+    elif kind == "large":
+        logits = 2.0e4 + rng.standard_normal((b, V)) * 3.0
+    else:
+        logits = rng.standard_normal((b, V))
+        logits[:, rng.integers(0, V, b)] += 12.0
+    logits = logits.astype(np.float32)
+    ids = rng.integers(0, 4096, b).astype(np.int32)
+    steps = rng.integers(0, 3000, b).astype(np.int32)
+    seed = int(rng.integers(0, 2 ** 63))
+    out = torch.zeros(b, dtype=torch.int32, device="cuda")
+    for T in (1.0, 0.7):
+        sr.sr_k_sample(dev(logits), V, b, V, dev(ids), dev(steps), seed, T, 1.0, 0, out)
+        want = [osamp.sample_token(logits[r], seed, int(ids[r]), int(steps[r]), T, 1.0, 0) for r in range(b)]
+        assert out.cpu().numpy().tolist() == want
+
+
 def test_gumbel_noise_bit_exact(sr):
     """With all logits equal to zero and T = 1 the argmax is the argmax of the noise itself."""
     V, b = 4099, 64

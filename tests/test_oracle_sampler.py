@@ -95,3 +95,18 @@ def test_ties_and_nan():
     z = perturbed_logits(np.array([2.0, 4.0], np.float32), 3, 0, 0, 2.0, 0.0, 0)
     g = gumbel_noise(3, 0, 0, 2)
     assert np.array_equal(z, (np.array([1.0, 2.0], np.float32) + g).astype(np.float32))
+
+
+def test_gumbel_noise_bound_for_skip_test():
+    """The sampler kernel skips an id whose uniform satisfies 1 - u > exp(ap - best + margin), margin >= 1e-4: valid
+    because the Gumbel noise as computed (two series logarithms) never exceeds -ln(1 - u) by 1e-5.  Checked over
+    every one of the 2^23 uniforms the generator can produce."""
+    w = np.arange(1 << 23, dtype=np.uint32)
+    u = (w.astype(np.float32) + np.float32(0.5)) * np.float32(2.0 ** -23)
+    g = -flog(-flog(u)).astype(np.float64)                      # the sampler's noise, as the kernel computes it
+    one_minus_u = ((np.uint32(0x7FFFFF) - w).astype(np.float32) + np.float32(0.5)) * np.float32(2.0 ** -23)
+    assert np.array_equal(one_minus_u.astype(np.float64), 1.0 - u.astype(np.float64))   # exact in float32
+    bound = -np.log(one_minus_u.astype(np.float64))             # g(u) <= -ln(1 - u) since -ln u >= 1 - u
+    assert np.max(g - bound) < 1e-5
+    exact = -np.log(-np.log(u.astype(np.float64)))
+    assert np.max(np.abs(g - exact)) < 1e-5 and np.max(np.abs(g)) < 17.0
