@@ -280,6 +280,18 @@ sr_status sr_k_sample(const float* logits, long long ld, int b, int vocab, const
                       int32_t* tokens_out, void* stream,
                       double* logprob_sum);
 
+/* LM head fused with sampling (Section 3 sampling step, as sr_k_sample, without storing logits):
+ * token[r] = the Gumbel-max sample of sr_k_sample over logits[r][v] = x[r] . W[v] (fp32 accumulation of
+ * `dtype` operands, SR_DT_F16 or SR_DT_BF16), with step = lens[orig_ids[r]] as the token index of the noise.
+ * x [M][K], W [vocab][K] (device, 16-byte aligned), K % 8 == 0, vocab % 32 == 0.  The GEMM's epilogue
+ * reduces each row's 64-id chunks to a 32-byte record; a second kernel picks the token.  The token equals
+ * sr_k_sample's on the logits sr_k_gemm (epilogue 0) computes with the same tile configuration: 256 x 256
+ * CTA-pair tiles from 512 rows, 128 x 256 tiles below.  Allocates M * ceil(vocab / 64) * 32 bytes of
+ * workspace on `stream` for the call. */
+sr_status sr_k_lm_head_sample(int dtype, const void* x, const void* W, int M, int vocab, int K,
+                              const int32_t* orig_ids, const int32_t* lens, uint64_t seed, float temperature,
+                              float eos_bias, int eos_id, int32_t* tokens_out, void* stream);
+
 /* r_cut selection (Eqs. cutoff.threshold, accepted.set) on b <= 4096 fp32
  * rewards: k = min(floor(alpha b), b - 1) (or k_override >= 0); r_cut = k-th
  * smallest by radix select on order-preserving keys; mask[i] = rewards[i] >= r_cut. */

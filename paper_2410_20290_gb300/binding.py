@@ -91,6 +91,7 @@ _SIG = {
     "sr_batch_query": [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P],
     "sr_batch_end": [_P, _P],
     "sr_k_sample": [_P, ctypes.c_longlong, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P, _P],
+    "sr_k_lm_head_sample": [_I, _P, _P, _I, _I, _I, _P, _P, ctypes.c_uint64, _F, _F, _I, _P, _P],
     "sr_set_reward": [_P, _I],
     "sr_set_rm_cache": [_P, ctypes.c_size_t],
     "sr_auto_b_init": [_P, ctypes.c_size_t, _I, _I, _I, _P],
@@ -290,6 +291,12 @@ def sr_k_sample(logits, ld, b, vocab, orig_ids, steps, seed, temperature, eos_bi
                 logprob_sum=None):
     _check(LIB.sr_k_sample(_ptr(logits), ld, b, vocab, _ptr(orig_ids), _ptr(steps), seed, temperature, eos_bias,
                            eos_id, _ptr(tokens_out), _stream(stream), _ptr(logprob_sum)))
+
+
+def sr_k_lm_head_sample(dtype, x, W, M, vocab, K, orig_ids, lens, seed, temperature, eos_bias, eos_id, tokens_out,
+                        stream=None):
+    _check(LIB.sr_k_lm_head_sample(dtype, _ptr(x), _ptr(W), M, vocab, K, _ptr(orig_ids), _ptr(lens), seed, temperature,
+                                   eos_bias, eos_id, _ptr(tokens_out), _stream(stream)))
 
 
 def sr_k_rcut(rewards, b, alpha, k_override, r_cut_out, mask_out, stream=None):

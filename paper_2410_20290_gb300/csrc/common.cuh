@@ -162,6 +162,22 @@ enum Epi { EPI_F32 = 0, EPI_ADD_F32 = 1, EPI_STORE = 2, EPI_SWIGLU = 3, EPI_GEGL
 
 // gemm_tc.cu: tcgen05 GEMM, C = A W^T, A and W both bf16 or both fp16 (et = SR_DT_BF16 / SR_DT_F16).
 sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, int K, int epi, cudaStream_t st);
+
+// One record of the LM head's sampling epilogue: row r, vocabulary ids 64 c .. 64 c + 63.  z = the largest
+// perturbed logit (-inf if none was finite), id its vocabulary id (INT_MAX if none), a its raw logit, (m, s) the
+// log-sum-exp partial of the raw logits (running max, sum of exp(logit - m)), a0 = id 0's raw logit (chunk 0).
+struct SampleRec {
+  float z;
+  int id;
+  float a, m, s, a0, pad0, pad1;
+};
+constexpr int SAMPLE_CHUNK = 64;
+// gemm_tc.cu: logits = x W^T for M rows and V vocabulary ids (fp16 or, bf, bf16 operands, fp32 accumulators) reduced to
+// SampleRec[M][ceil(V / 64)] in the GEMM's epilogue -- the logits are never stored.  Row r's noise is keyed on
+// (seed, ids[r], lens[ids[r]]); lp != 0 adds the log-sum-exp partials.
+sr_status lm_head_sample(bool bf, const void* x, const void* W, int M, int V, int K, const int* ids, const int* lens,
+                         uint64_t seed, float temperature, float eos_bias, int eos_id, int lp, SampleRec* rec,
+                         cudaStream_t st);
 // gemm_f32.cu: fp32 SIMT GEMM (epilogues EPI_F32, EPI_ADD_F32, EPI_STORE).
 sr_status gemm_f32(const float* A, const float* W, float* C, int M, int N, int K, int epi, cudaStream_t st);
 
@@ -193,6 +209,10 @@ sr_status launch_sample(const float* logits, long long ld, int b, int V, const i
                         int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st,
                         double* lp_sum = nullptr,   // lp_sum: += ln p(token) per candidate id (Section 5.3 reward)
                         const int* n_rows = nullptr);  // device count: rows >= *n_rows are skipped
+// The same decision from lm_head_sample's records (n_chunks per row), reduced in vocabulary order.
+sr_status launch_sample_reduce(const SampleRec* rec, int n_chunks, int b, const int* orig_ids, int eos_id,
+                               int* tokens_out, int* tok_hist, int max_new, int* lens, int* status, cudaStream_t st,
+                               double* lp_sum = nullptr, const int* n_rows = nullptr);
 
 // attention.cu
 // Workspace of the streaming decode-attention kernel (16-bit KV, head_dim 128, 8 kv heads): one persistent

@@ -36,6 +36,7 @@
 #include <type_traits>
 
 #include "common.cuh"
+#include "sampling.cuh"
 #include "tma.cuh"
 
 namespace sr {
@@ -53,9 +54,13 @@ struct Cfg {
   static constexpr int A_BYTES = TM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (192 * 1024) / STAGE_BYTES;  // 4 / 6 / 8 for BN 256 / 128 / 64; 3 for 256 x 256
+  static constexpr int STAGES = (200 * 1024) / STAGE_BYTES;  // 4 / 5 / 6 / 8 for BN 256 / 192 / 128 / 64; 3 for 256 x 256
   static constexpr int NACC = (MH * BN * 2 <= 512) ? 2 : 1;   // accumulator buffers in TMEM
-  static constexpr int TMEM_COLS = NACC * MH * BN;
+  static constexpr int TMEM_USED = NACC * MH * BN;
+  // tcgen05.alloc takes a power of two of at least 32 columns (384 for two BN = 192 accumulators -> 512)
+  static constexpr int TMEM_COLS = TMEM_USED <= 32 ? 32 : TMEM_USED <= 64 ? 64 : TMEM_USED <= 128 ? 128
+                                 : TMEM_USED <= 256 ? 256 : 512;
+  static_assert(TMEM_USED <= 512, "accumulators exceed TMEM");
   static constexpr int EPI_WARPS = 4 * MH;
   static constexpr int THREADS = 64 + 32 * EPI_WARPS;
   static constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
@@ -108,6 +113,14 @@ struct EpiArgs {
   int ldo;  // elements
   int kind;
   int bf;   // operands and 16-bit outputs are bf16 (1) or fp16 (0)
+  // sampling epilogue (LM head): one SampleRec per row and 64 vocabulary ids, [rows][n_chunks]; each row's
+  // candidate id and token count select its noise
+  SampleRec* rec;
+  int n_chunks;
+  const int* ids;
+  const int* lens;
+  GumbelParams gp;
+  int lp;  // also the log-sum-exp of the raw logits (self-likelihood reward)
 };
 
 // ---- CTA-pair (cta_group::2) forms ----
@@ -219,15 +232,115 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& ep, float* v, int row, 
   }
 }
 
-// Epilogue of one accumulator row segment: this thread's row of BNC fp32 columns at TMEM address `tbase`,
-// 64 columns per load and wait.
+// Sampling epilogue of the LM head (fused next-token sampling): the logits of one row are never stored; the
+// Gumbel-max scan of sampling.cuh runs over them in id order (Philox counters of 4 ids, the exact skip test) and
+// the row's record for each 64-id chunk keeps the largest perturbed logit, its id and raw logit, and the chunk's
+// log-sum-exp partial.  The values are the same fp32 accumulators the plain epilogue would store, so the sampled
+// token equals k_sample's on stored logits.  TMEM is read 16 columns at a time in a loop that is not unrolled,
+// which keeps the epilogue's code small next to the MMA and TMA warps it shares the SM with.
+struct SampleState {
+  float best, best_a, m, s;
+  int best_v;
+};
+
+__device__ __forceinline__ void sample_reset(SampleState& q) {
+  q.best = -__int_as_float(0x7f800000), q.best_a = 0.f, q.m = -__int_as_float(0x7f800000), q.s = 0.f;
+  q.best_v = 0x7fffffff;
+}
+
+// ids col .. col+31 (col a multiple of 32), v their 32 logits.  The eight Philox calls are independent (eight
+// dependency chains in flight: the epilogue has one warp per SMSP, so this is its only latency hiding); the
+// skip tests run against `ref`, the row's best before these ids (never above the running best, so a skipped id
+// still cannot win), and are independent too; the ids that pass are then scanned in order.
+__device__ __forceinline__ void sample_piece(const EpiArgs& ep, const float* v, int col, int N, int id, int step,
+                                             SampleState& q) {
+  uint32_t words[32];
+#pragma unroll
+  for (int g4 = 0; g4 < 8; ++g4) {
+    const uint4 w = philox4x32_10(make_uint4((uint32_t)((col >> 2) + g4), (uint32_t)id, (uint32_t)step, 0u),
+                                  ep.gp.k0, ep.gp.k1);
+    words[4 * g4] = w.x, words[4 * g4 + 1] = w.y, words[4 * g4 + 2] = w.z, words[4 * g4 + 3] = w.w;
+  }
+  const float ref = q.best;
+  uint32_t pass = 0u;
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (col + j < N && !gumbel_skip(v[j], col + j, words[j], ep.gp, ref)) pass |= 1u << j;
+  if (ep.lp) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (col + j < N) lse_step(v[j], q.m, q.s);
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if ((pass >> j) & 1u)
+      if (gumbel_step(v[j], col + j, words[j], ep.gp, q.best, q.best_v)) q.best_a = v[j];
+}
+
+__device__ __forceinline__ void sample_record(const EpiArgs& ep, const SampleState& q, int row, int col, float a0) {
+  float4* dst = reinterpret_cast<float4*>(ep.rec + (size_t)row * ep.n_chunks + col / 64);
+  dst[0] = make_float4(q.best, __int_as_float(q.best_v), q.best_a, q.m);
+  dst[1] = make_float4(q.s, a0, 0.f, 0.f);  // a0: id 0's raw logit in chunk 0 (the all -inf fallback)
+}
+
+// A 64-column chunk already in registers (the stream-K merge path).
+__device__ __forceinline__ void sample_chunk(const EpiArgs& ep, const float* v, int row, int col, int M, int N) {
+  if (row >= M || col >= N) return;
+  const int id = ep.ids[row];
+  const int step = ep.lens[id];
+  SampleState q;
+  sample_reset(q);
+#pragma unroll
+  for (int p = 0; p < 64; p += 32) sample_piece(ep, v + p, col + p, N, id, step, q);
+  sample_record(ep, q, row, col, v[0]);
+}
+
+// The sampling epilogue of one accumulator row segment of BNC columns at TMEM address `tbase`.
 template <int BNC>
-__device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int row, int col0, int M, int N) {
+__device__ __forceinline__ void sample_store(const EpiArgs& ep, uint32_t tbase, int row, int col0, int M, int N) {
+  const bool live = row < M;
+  const int id = live ? ep.ids[row] : 0;
+  const int step = live ? ep.lens[id] : 0;
+  // The scan of each chunk starts from the best of the tile's earlier chunks: an id not above it cannot win, and
+  // a chunk whose record keeps that value carries no id (INT_MAX), which never wins the reduction's comparisons.
+  float carry = -__int_as_float(0x7f800000);
 #pragma unroll 1
   for (int c = 0; c < BNC; c += 64) {
-    float v[64];
-    tmem_ld64(tbase + c, v);
-    epi_chunk(ep, v, row, col0 + c, M, N);
+    float w64[64];
+    tmem_ld64(tbase + c, w64);  // warp-collective: every lane loads
+    SampleState q;
+    sample_reset(q);
+    q.best = carry;
+#pragma unroll 1
+    for (int p = 0; p < 2; ++p) {
+      float v[32];
+      if (p == 0) {  // static register indices for the half
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = w64[j];
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = w64[32 + j];
+      }
+      if (live && col0 + c + 32 * p < N) sample_piece(ep, v, col0 + c + 32 * p, N, id, step, q);
+    }
+    if (live && col0 + c < N) sample_record(ep, q, row, col0 + c, w64[0]);
+    carry = q.best;
+  }
+}
+
+// Epilogue of one accumulator row segment: this thread's row of BNC fp32 columns at TMEM address `tbase`,
+// 64 columns per load and wait.  EK = 1: the sampling epilogue.
+template <int BNC, int EK = 0>
+__device__ __forceinline__ void epi_store(const EpiArgs& ep, uint32_t tbase, int row, int col0, int M, int N) {
+  if constexpr (EK == 1) {
+    sample_store<BNC>(ep, tbase, row, col0, M, N);
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < BNC; c += 64) {
+      float v[64];
+      tmem_ld64(tbase + c, v);
+      epi_chunk(ep, v, row, col0 + c, M, N);
+    }
   }
 }
 
@@ -281,7 +394,7 @@ __device__ __forceinline__ bool sk_segment(bool on, int i, int num_tiles, int nu
   return true;
 }
 
-template <int TM, int BN>
+template <int TM, int BN, int EK = 0>
 __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
               int N, int K, int* err, unsigned long long wait_ns, SkArgs sk) {
@@ -449,7 +562,7 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
       const int row = mb * TM + half * BM + quad * 32 + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * ACC_COLS + half * BN);
       if (sg.kb0 == 0 && sg.kb1 == num_k) {
-        epi_store<BN>(ep, tbase, row, nb * BN, M, N);
+        epi_store<BN, EK>(ep, tbase, row, nb * BN, M, N);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -499,7 +612,10 @@ __global__ void __launch_bounds__(Cfg<TM, BN>::THREADS, 1)
             v[4 * q] += p.x, v[4 * q + 1] += p.y, v[4 * q + 2] += p.z, v[4 * q + 3] += p.w;
           }
         }
-        epi_chunk(ep, v, row, nb * BN + c, M, N);
+        if constexpr (EK == 1)
+          sample_chunk(ep, v, row, nb * BN + c, M, N);
+        else
+          epi_chunk(ep, v, row, nb * BN + c, M, N);
       }
       if (lane == 0) sk.cnt[(size_t)tile * 4 + quad] = 0;
     }
@@ -542,7 +658,7 @@ __host__ __device__ constexpr uint32_t idesc_pair(bool bf, int N) {
          ((uint32_t)(256 >> 4) << 24);
 }
 
-template <int BNP>
+template <int BNP, int EK = 0>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     k_gemm_pair(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, EpiArgs ep, int M,
                 int N, int K, int* err) {
@@ -697,7 +813,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       tc_fence_after();
       const int row = mb * 256 + (int)rank * BM + quad * 32 + lane;
       const uint32_t tbase = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BNP);
-      epi_store<BNP>(ep, tbase, row, nb * BNP, M, N);
+      epi_store<BNP, EK>(ep, tbase, row, nb * BNP, M, N);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cta(&tempty[acc], 0);
@@ -1030,10 +1146,10 @@ int* g_err = nullptr;
 // traffic, pipeline fill, epilogue) that a sweep of the decode and scoring shapes on GB300 puts
 // at about the cost of 430 columns of a K = 4096 tile.
 int pick_bn(int M, int N, int K) {
-  if (g_bn_override == 64 || g_bn_override == 128 || g_bn_override == 256) return g_bn_override;
+  if (g_bn_override == 64 || g_bn_override == 128 || g_bn_override == 192 || g_bn_override == 256) return g_bn_override;
   int best = 256;
   double best_cost = -1;
-  for (int bn : {256, 128, 64}) {
+  for (int bn : {256, 192, 128, 64}) {
     const long long tiles = (long long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
     const long long waves = (tiles + g_num_sms - 1) / g_num_sms;
     const double cost = (double)waves * (bn * (K / 4096.0) + 430.0);
@@ -1092,13 +1208,13 @@ sr_status sk_workspace(size_t part_floats, size_t cnt_ints, cudaStream_t st, SkA
   return SR_OK;
 }
 
-template <int TM, int BN>
+template <int TM, int BN, int EK = 0>
 sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
                     cudaStream_t st, bool streamk = false) {
   using C = Cfg<TM, BN>;
   static int max_ctas = 0;
   if (!max_ctas) {
-    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
+    SR_CUDA(cudaFuncSetAttribute(k_gemm_tc<TM, BN, EK>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
     max_ctas = g_num_sms;
   }
   const int tiles = ((M + TM - 1) / TM) * ((N + BN - 1) / BN);
@@ -1109,7 +1225,7 @@ sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs&
     grid = max_ctas;
     SR_TRY(sk_workspace((size_t)grid * 2 * TM * BN, (size_t)tiles * 4, st, &sk));
   }
-  launch_k(k_gemm_tc<TM, BN>, grid, C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err, g_wait_ns, sk);
+  launch_k(k_gemm_tc<TM, BN, EK>, grid, C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err, g_wait_ns, sk);
   SR_CUDA(cudaGetLastError());
   return SR_OK;
 }
@@ -1119,29 +1235,33 @@ sr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs&
 // K >= 8192) below 8192 rows; at least two pair rows (M >= 512) so the 256-row tiles are not mostly padding.
 bool pick_pair(int M, int N, int K, bool gated) {
   if (M < 512) return false;
+  // gated shapes: only where padding M to 256-row pair tiles wastes no more rows than 128-row tiles (at 600 rows
+  // the pair ran 161 us against 139 us on 128 x 256 tiles for 28672 x 4096)
+  const double eff_pair = (double)M / (256.0 * ((M + 255) / 256)), eff_128 = (double)M / (128.0 * ((M + 127) / 128));
+  if (gated && eff_pair + 0.02 < eff_128) return false;
   return gated || N >= 65536 || (N <= 4096 && K >= 8192 && M < 8192);
 }
 
-template <int BNP>
+template <int BNP, int EK = 0>
 sr_status launch_pair(const CUtensorMap& ta, const CUtensorMap& tb, const EpiArgs& ep, int M, int N, int K,
                       cudaStream_t st) {
   using C = PairCfg<BNP>;
   static int max_pairs = 0;
   if (!max_pairs) {
-    SR_CUDA(cudaFuncSetAttribute(k_gemm_pair<BNP>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
+    SR_CUDA(cudaFuncSetAttribute(k_gemm_pair<BNP, EK>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
     max_pairs = g_num_sms / 2;
     cudaLaunchConfig_t qc = {};
     qc.gridDim = dim3(max_pairs * 2);
     qc.blockDim = dim3(C::THREADS);
     qc.dynamicSmemBytes = C::SMEM_BYTES;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, k_gemm_pair<BNP>, &qc) == cudaSuccess && clusters > 0)
+    if (cudaOccupancyMaxActiveClusters(&clusters, k_gemm_pair<BNP, EK>, &qc) == cudaSuccess && clusters > 0)
       max_pairs = std::min(max_pairs, clusters);
     cudaGetLastError();
   }
   const int tiles = ((M + 255) / 256) * ((N + BNP - 1) / BNP);
   const int pairs = std::min(tiles, max_pairs);
-  launch_k(k_gemm_pair<BNP>, pairs * 2, C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err);
+  launch_k(k_gemm_pair<BNP, EK>, pairs * 2, C::THREADS, C::SMEM_BYTES, st, ta, tb, ep, M, N, K, g_err);
   SR_CUDA(cudaGetLastError());
   return SR_OK;
 }
@@ -1270,14 +1390,8 @@ sr_status encode_kmajor(CUtensorMap* map, const void* base, bool bf, int rows, i
 
 }  // namespace
 
-sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, int K, int epi, cudaStream_t st) {
-  if (et != SR_DT_BF16 && et != SR_DT_F16) return set_err(SR_ERR_INVALID_ARG, "gemm: operands must be bf16 or fp16");
-  const bool bf = et == SR_DT_BF16;
-  if (M <= 0 || N <= 0 || K <= 0) return M == 0 ? SR_OK : set_err(SR_ERR_INVALID_ARG, "gemm: bad shape");
-  if (K % 8 != 0 || N % 32 != 0 || ((epi == EPI_SWIGLU || epi == EPI_GEGLU) && N % 64 != 0))
-    return set_err(SR_ERR_INVALID_ARG, "gemm: needs K %% 8 == 0 and N %% 32 == 0 (N %% 64 for gated)");
-  if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15)
-    return set_err(SR_ERR_INVALID_ARG, "gemm: operands must be 16-byte aligned");
+// SM count, the error word and the tuning switches, on the first GEMM of the process.
+sr_status gemm_init() {
   if (!g_num_sms) {
     int dev;
     SR_CUDA(cudaGetDevice(&dev));
@@ -1290,6 +1404,18 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
     if (const char* e = getenv("SR_GEMM_WAIT_NS")) g_wait_ns = strtoull(e, nullptr, 10);
     if (const char* e = getenv("SR_GEMM_STREAMK")) g_sk_override = atoi(e);
   }
+  return SR_OK;
+}
+
+sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, int K, int epi, cudaStream_t st) {
+  if (et != SR_DT_BF16 && et != SR_DT_F16) return set_err(SR_ERR_INVALID_ARG, "gemm: operands must be bf16 or fp16");
+  const bool bf = et == SR_DT_BF16;
+  if (M <= 0 || N <= 0 || K <= 0) return M == 0 ? SR_OK : set_err(SR_ERR_INVALID_ARG, "gemm: bad shape");
+  if (K % 8 != 0 || N % 32 != 0 || ((epi == EPI_SWIGLU || epi == EPI_GEGLU) && N % 64 != 0))
+    return set_err(SR_ERR_INVALID_ARG, "gemm: needs K %% 8 == 0 and N %% 32 == 0 (N %% 64 for gated)");
+  if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15)
+    return set_err(SR_ERR_INVALID_ARG, "gemm: operands must be 16-byte aligned");
+  SR_TRY(gemm_init());
   const bool gated = epi == EPI_SWIGLU || epi == EPI_GEGLU;
   CUtensorMap ta, tb;
   EpiArgs ep{C, gated ? N / 2 : N, epi, bf ? 1 : 0};
@@ -1316,7 +1442,39 @@ sr_status gemm_tc(int et, const void* A, const void* W, void* C, int M, int N, i
   if (tm == 256) return launch_bn<256, 256>(ta, tb, ep, M, N, K, st);
   if (bn == 64) return launch_bn<128, 64>(ta, tb, ep, M, N, K, st);
   if (bn == 128) return launch_bn<128, 128>(ta, tb, ep, M, N, K, st);
+  if (bn == 192) return launch_bn<128, 192>(ta, tb, ep, M, N, K, st);
   return launch_bn<128, 256>(ta, tb, ep, M, N, K, st);
+}
+
+// Fused LM head + sampling: 256 x 256 CTA-pair tiles from 512 rows (as the launcher picks for LM-head widths),
+// 128 x 256 one-SM tiles below; the sampling epilogue replaces the logits store.
+sr_status lm_head_sample(bool bf, const void* x, const void* W, int M, int V, int K, const int* ids, const int* lens,
+                         uint64_t seed, float temperature, float eos_bias, int eos_id, int lp, SampleRec* rec,
+                         cudaStream_t st) {
+  if (M <= 0) return M == 0 ? SR_OK : set_err(SR_ERR_INVALID_ARG, "lm_head_sample: bad shape");
+  if (V <= 0 || K <= 0 || K % 8 != 0 || V % 32 != 0)
+    return set_err(SR_ERR_INVALID_ARG, "lm_head_sample: needs K %% 8 == 0 and V %% 32 == 0");
+  if (!(temperature > 0.f)) return set_err(SR_ERR_INVALID_ARG, "temperature must be > 0");
+  if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) | reinterpret_cast<uintptr_t>(rec)) & 15)
+    return set_err(SR_ERR_INVALID_ARG, "lm_head_sample: operands must be 16-byte aligned");
+  SR_TRY(gemm_init());
+  EpiArgs ep{};
+  ep.kind = EPI_F32;  // unused by the sampling epilogue
+  ep.bf = bf ? 1 : 0;
+  ep.rec = rec;
+  ep.n_chunks = (V + SAMPLE_CHUNK - 1) / SAMPLE_CHUNK;
+  ep.ids = ids;
+  ep.lens = lens;
+  ep.gp = GumbelParams{(uint32_t)(seed & 0xFFFFFFFFu), (uint32_t)(seed >> 32), 1.0f / temperature, eos_bias, eos_id};
+  ep.lp = lp;
+  CUtensorMap ta, tb;
+  SR_TRY(encode_kmajor(&ta, x, bf, M, K, BM));
+  if (M >= 512) {
+    SR_TRY(encode_kmajor(&tb, W, bf, V, K, 128));
+    return launch_pair<256, 1>(ta, tb, ep, M, V, K, st);
+  }
+  SR_TRY(encode_kmajor(&tb, W, bf, V, K, 256));
+  return launch_bn<128, 256, 1>(ta, tb, ep, M, V, K, st);
 }
 
 // The device error word shared by the kernels with bounded waits (allocated on first use; nullptr when

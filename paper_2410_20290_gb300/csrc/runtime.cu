@@ -34,6 +34,18 @@ sr_status set_err(sr_status s, const char* fmt, ...) {
 int* gemm_error_word();
 void gemm_release_workspace(cudaStream_t st);
 
+// LM head and sampling fused (16-bit models), only with SR_FUSED_SAMPLE=1: on GB300 the fused epilogue's Gumbel
+// scan (a Philox call per 4 ids, one epilogue warp per SMSP) outlasts the GEMM's main loop, 1.63 against 1.10 ms
+// for the LM head plus the separate sampling pass at 1024 rows, so by default the logits are stored and sampled
+// in a pass of their own.
+bool fused_sample_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("SR_FUSED_SAMPLE");
+    return e && e[0] == '1';
+  }();
+  return on;
+}
+
 bool pdl_enabled() {
   static const bool on = [] {
     const char* e = getenv("SR_PDL");
@@ -521,6 +533,8 @@ struct sr_ctx {
       *prompt_row = nullptr, *ids = nullptr, *prompt = nullptr, *iota = nullptr, *meta = nullptr, *out_tok = nullptr,
       *last_row = nullptr;
   float *reward = nullptr, *rr = nullptr, *logits = nullptr, *logits0 = nullptr;
+  sr::SampleRec* srec = nullptr;  // records of the LM head's sampling epilogue, [live rows][vocab / 64]
+  size_t c_srec = 0;
   // self-likelihood reward (Section 5.3): running ln p(Y | X) per candidate id
   int reward_kind = SR_REWARD_MODEL;
   double* lp_sum = nullptr;
@@ -627,7 +641,6 @@ sr_status prepare_state(sr_ctx* c, sr_batch& b) {
   SR_TRY(grow(c->mask, c->c_mask, N));
   SR_TRY(grow(c->last_row, c->c_lastrow, N));
   SR_TRY(grow(c->out_tok, c->c_out, (size_t)b.max_new));
-  SR_TRY(grow(c->logits, c->c_logits, N * c->gen.d.vocab));
   SR_TRY(grow(c->logits0, c->c_logits0, (size_t)c->gen.d.vocab));
   SR_TRY(c->wg.ensure(c->gen, std::max<int>(b.N, b.P)));
   const int iota_n = std::max(c->gen.d.max_pos, c->rm.d.max_pos);
@@ -812,15 +825,29 @@ sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host, bool sync = tr
     Scope sc(pf, SR_KC_ELEMENTWISE, st);
     SR_TRY(launch_norm(m.et, d.norm, w.x, m.final_w, m.final_b, d.norm_eps, n, D, w.xn, st));
   }
-  SR_TRY(linear(m, w.xn, m.lm_head, c->logits, n, d.vocab, D, EPI_F32, st, pf, SR_KC_GEMM_DECODE));
-  if (logits_host)
-    SR_CUDA(cudaMemcpyAsync(logits_host, c->logits, (size_t)n * d.vocab * sizeof(float), cudaMemcpyDeviceToHost,
-                            st));
-  {
+  double* lp = b.reward_kind == SR_REWARD_LOGPROB ? c->lp_sum : nullptr;
+  if (m.et == SR_DT_F16 && !logits_host && fused_sample_enabled()) {
+    // LM head fused with sampling: the GEMM epilogue reduces each row's logits to one record per 64 ids
+    const int nch = (d.vocab + SAMPLE_CHUNK - 1) / SAMPLE_CHUNK;
+    SR_TRY(grow(c->srec, c->c_srec, (size_t)n * nch));
+    {
+      Scope sc(pf, SR_KC_GEMM_DECODE, st, 2.0 * n * d.vocab * D,
+               m.esz * ((double)n * D + (double)d.vocab * D) + sizeof(SampleRec) * (double)n * nch);
+      SR_TRY(lm_head_sample(false, w.xn, m.lm_head, n, d.vocab, D, c->live, c->len, b.seed, b.temperature,
+                            b.eos_bias, b.eos_id, lp ? 1 : 0, c->srec, st));
+    }
+    Scope sc(pf, SR_KC_SAMPLE, st, 0, sizeof(SampleRec) * (double)n * nch);
+    SR_TRY(launch_sample_reduce(c->srec, nch, n, c->live, b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status,
+                                st, lp, c->ctrl + C_NLIVE));
+  } else {
+    SR_TRY(grow(c->logits, c->c_logits, (size_t)n * d.vocab));
+    SR_TRY(linear(m, w.xn, m.lm_head, c->logits, n, d.vocab, D, EPI_F32, st, pf, SR_KC_GEMM_DECODE));
+    if (logits_host)
+      SR_CUDA(cudaMemcpyAsync(logits_host, c->logits, (size_t)n * d.vocab * sizeof(float), cudaMemcpyDeviceToHost,
+                              st));
     Scope sc(pf, SR_KC_SAMPLE, st, 0, 4.0 * n * d.vocab);
     SR_TRY(launch_sample(c->logits, d.vocab, n, d.vocab, c->live, nullptr, b.seed, b.temperature, b.eos_bias,
-                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, st,
-                         b.reward_kind == SR_REWARD_LOGPROB ? c->lp_sum : nullptr, c->ctrl + C_NLIVE));
+                         b.eos_id, nullptr, c->tok, b.max_new, c->len, c->status, st, lp, c->ctrl + C_NLIVE));
   }
   {
     Scope sc(pf, SR_KC_CONTROL, st);
@@ -1311,7 +1338,7 @@ void sr_destroy(sr_ctx* c) {
   void* dev[] = {c->pool, c->rm_pk, c->rm_pv, c->rm_pool, c->rm_pt, c->row_cand, c->len, c->status, c->tok, c->pt, c->live, c->rset, c->free_stack,
                  c->tok_in, c->pos_in, c->kv_len, c->tail_dst, c->prompt_row, c->ids, c->prompt, c->iota, c->meta,
                  c->out_tok, c->last_row, c->reward, c->rr, c->logits, c->logits0, c->mask, c->ctrl, c->ctrlf, c->d_score,
-                 c->d_outlen};
+                 c->d_outlen, c->srec};
   for (void* p : dev)
     if (p) cudaFree(p);
   if (c->h_ctrl) cudaFreeHost(c->h_ctrl);
@@ -1525,6 +1552,27 @@ sr_status sr_k_sample(const float* logits, long long ld, int b, int vocab, const
     return set_err(SR_ERR_INVALID_ARG, "sr_k_sample: bad argument");
   return launch_sample(logits, ld, b, vocab, orig_ids, steps, seed, temperature, eos_bias, eos_id, tokens_out,
                        nullptr, 0, nullptr, nullptr, static_cast<cudaStream_t>(stream), logprob_sum);
+}
+
+sr_status sr_k_lm_head_sample(int dtype, const void* x, const void* W, int M, int vocab, int K,
+                              const int32_t* orig_ids, const int32_t* lens, uint64_t seed, float temperature,
+                              float eos_bias, int eos_id, int32_t* tokens_out, void* stream) {
+  if (!x || !W || !orig_ids || !lens || !tokens_out || M < 0 || vocab < 1)
+    return set_err(SR_ERR_INVALID_ARG, "sr_k_lm_head_sample: bad argument");
+  if (dtype != SR_DT_F16 && dtype != SR_DT_BF16)
+    return set_err(SR_ERR_INVALID_ARG, "sr_k_lm_head_sample: dtype must be SR_DT_F16 or SR_DT_BF16");
+  if (M == 0) return SR_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int nch = (vocab + SAMPLE_CHUNK - 1) / SAMPLE_CHUNK;
+  SampleRec* rec = nullptr;
+  SR_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&rec), (size_t)M * nch * sizeof(SampleRec), st));
+  sr_status s = lm_head_sample(dtype == SR_DT_BF16, x, W, M, vocab, K, orig_ids, lens, seed, temperature, eos_bias,
+                               eos_id, 0, rec, st);
+  if (s == SR_OK)
+    s = launch_sample_reduce(rec, nch, M, orig_ids, eos_id, tokens_out, nullptr, 0, const_cast<int*>(lens), nullptr,
+                             st);
+  cudaFreeAsync(rec, st);
+  return s;
 }
 
 sr_status sr_k_rcut(const float* rewards, int b, float alpha, int k_override, float* r_cut_out, uint8_t* mask_out,

@@ -5,6 +5,7 @@
   python -m paper_2410_20290_gb300.microbench prefill_attn n_seq tau n_pre Hq Hkv dh
   python -m paper_2410_20290_gb300.microbench sample b V
   python -m paper_2410_20290_gb300.microbench decode_gemms M
+  python -m paper_2410_20290_gb300.microbench lm_head_sample M V K
 
 Prints one JSON line with the mean launch time and the achieved rate (TFLOP/s or GB/s) of the
 algorithmic work.  Operands are sized by the shape given; choose shapes larger than the 129 MB L2
@@ -94,6 +95,25 @@ def sample(b, V, iters=20):
     return dict(kernel="sample", b=b, V=V, ms=ms, gbs=b * V * 4 / ms / 1e6)
 
 
+def lm_head_sample(M, V, K, iters=10):
+    """The LM head fused with sampling (sr_k_lm_head_sample) against the LM-head GEMM storing fp32 logits followed
+    by the sampling pass over them (sr_k_gemm + sr_k_sample)."""
+    g = torch.Generator(device="cuda").manual_seed(0)
+    x = (torch.randn(M, K, device="cuda", generator=g) / K ** 0.5).to(torch.float16)
+    W = torch.randn(V, K, device="cuda", generator=g).to(torch.float16)
+    ids = torch.arange(M, device="cuda", dtype=torch.int32)
+    lens = torch.full((max(M, 1),), 100, device="cuda", dtype=torch.int32)
+    tok = torch.zeros(M, device="cuda", dtype=torch.int32)
+    logits = torch.zeros(M, V, device="cuda")
+    s = torch.cuda.current_stream().cuda_stream
+    fused = _time(lambda: sr.sr_k_lm_head_sample(DT_F16, x, W, M, V, K, ids, lens, 7, 1.0, 1.0, 0, tok, s), iters)
+    gemm = _time(lambda: sr.sr_k_gemm(DT_F16, x, W, logits, M, V, K, 0, s), iters)
+    samp = _time(lambda: sr.sr_k_sample(logits, V, M, V, ids, lens, 7, 1.0, 1.0, 0, tok, s), iters)
+    fl = 2.0 * M * V * K
+    return dict(kernel="lm_head_sample", M=M, V=V, K=K, fused_ms=fused, gemm_ms=gemm, sample_ms=samp,
+                unfused_ms=gemm + samp, fused_tflops=fl / fused / 1e9)
+
+
 def decode_gemms(M, iters=5):
     """The five GEMMs of one decode step of the Llama-3-8B-shaped generator at M live rows (QKV, O + residual,
     gate/up + SwiGLU, down + residual, LM head), each launched `iters` times; per shape the mean time and the
@@ -112,7 +132,7 @@ def decode_gemms(M, iters=5):
 def main(argv):
     kind, nums = argv[0], [int(x) for x in argv[1:]]
     fn = {"gemm": gemm, "decode_attn": decode_attn, "prefill_attn": prefill_attn, "sample": sample,
-          "decode_gemms": decode_gemms}[kind]
+          "decode_gemms": decode_gemms, "lm_head_sample": lm_head_sample}[kind]
     print(json.dumps(fn(*nums)), flush=True)
 
 

@@ -20,6 +20,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 @pytest.mark.parametrize("env", [{"SR_GEMM_SKINNY": "0"}, {"SR_GEMM_SKINNY": "1"}, {"SR_GEMM_PAIR": "1"},
                                  {"SR_GEMM_TM": "256"}, {"SR_GEMM_BN": "64"}, {"SR_GEMM_BN": "128"},
+                                 {"SR_GEMM_BN": "192"},
                                  {"SR_GEMM_STREAMK": "1"}])
 def test_gemm_tile_variant(env):
     child = dict(os.environ, **env)
