@@ -71,3 +71,27 @@ def test_host_only_entry_points_validate_arguments(lib_path):
         assert e.value.status == b.SR_ERR_INVALID_ARG
     assert b.sr_auto_b_init(m, 1000, 16, 8, 16) == 0          # a pool below one page: nothing fits (SR_ERR_OOM)
     assert "tau_min" in b.LIB.sr_last_error().decode()
+
+
+def test_kernel_entry_points_reject_bad_arguments_on_the_host(lib_path):
+    """The kernel-level calls check pointers, dtypes and epilogue codes before any device work, so a caller's
+    mistake is an SR_ERR_INVALID_ARG status (with a message), never a launch on bad arguments.  The host arrays
+    passed here are never dereferenced: every call returns at its argument check."""
+    import numpy as np
+    from paper_2410_20290_gb300 import binding as b
+    import sr_inputs as si
+    x = np.zeros(64, np.float32)
+    ids = np.zeros(4, np.int32)
+    cases = [
+        lambda: b.sr_k_lm_head_sample(si.DT_F16, None, x, 4, 64, 16, ids, ids, 1, 1.0, 0.0, 0, ids),
+        lambda: b.sr_k_lm_head_sample(si.DT_F32, x, x, 4, 64, 16, ids, ids, 1, 1.0, 0.0, 0, ids),   # 16-bit only
+        lambda: b.sr_k_sample(None, 64, 4, 64, ids, ids, 1, 1.0, 0.0, 0, ids),
+        lambda: b.sr_k_gemm(si.DT_F16, None, x, x, 4, 64, 16, 0),
+        lambda: b.sr_k_gemm(si.DT_F16, x, x, x, 4, 64, 16, 9),                                     # no epilogue 9
+        lambda: b.sr_k_decode_attention(si.DT_F16, None, x, ids, 1, ids, ids, 4, 32, 8, 128, 0, x),
+    ]
+    for call in cases:
+        with pytest.raises(b.SrError) as e:
+            call()
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        assert b.LIB.sr_last_error().decode()
