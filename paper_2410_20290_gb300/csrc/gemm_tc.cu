@@ -7,22 +7,25 @@
 // tensor memory.
 //
 // Design (persistent, warp-specialised, one CTA per SM):
-//   warp 0      : TMA producer -- 128x64 A and BNx64 W tiles (BN = 256, 128 or 64, chosen per
-//                 shape so the tile count fills the SMs), 128-byte swizzle, STAGES-deep ring
-//                 (~192 KB of shared memory in flight per SM)
+//   warp 0      : TMA producer -- 128x64 A and BNx64 W tiles (BN = 256, 192, 128 or 64, chosen per
+//                 shape by a waves x per-tile-cost model), 128-byte swizzle, STAGES-deep ring
+//                 (up to 200 KB of shared memory in flight per SM)
 //   warp 1      : allocates 2*BN TMEM columns; one elected lane issues tcgen05.mma (M=128, N=BN,
 //                 K=16) and tcgen05.commit to release smem stages / publish accumulators
 //   warps 2..5  : epilogue -- tcgen05.ld 32 lanes x 64 columns per warp and wait (the warp's TMEM
 //                 lane quadrant is warp % 4), fused conversion / residual add / gated activation,
 //                 direct global stores
 // Two BN-column accumulators let the epilogue of tile i overlap the mainloop of tile i+1.
-// Tiles are walked M-fastest so that the CTAs running at the same time share W tiles in L2.
+// Tiles are walked in groups of 16 M tiles, M fastest within a group, so that the CTAs running at the same
+// time share W tiles and one band of A rows in L2.
 // Two variants raise the MMA work per staged byte (the limit of the 128-row tiles on GB300):
 // 256 x 256 tiles on one SM (two M = 128 MMAs per W tile, single-buffered accumulator), and
 // 256 x 256 tiles on a CTA pair (cta_group::2, M = 256 MMAs, each SM staging half of A and W,
 // double-buffered accumulators).  Decode batches of at most 512 rows can instead run the product
 // transposed (C^T = W A^T) on a CTA pair, every activation row on the MMA's N side, with the K range
 // split over the SMs and the fp32 partials summed in slice order.  The launcher picks per shape.
+// Opt-in forms: stream-K shares of k-blocks on 128 x 256 tiles (SR_GEMM_STREAMK=1), and the LM head's
+// sampling epilogue (EK = 1: Gumbel-max records instead of stored logits, sampling.cuh).
 // Every mbarrier wait is bounded (about 2 s of %globaltimer); on expiry the CTA records an error,
 // drains its own TMA copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
