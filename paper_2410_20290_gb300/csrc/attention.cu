@@ -3,7 +3,14 @@
 // softmax(q k^T / sqrt(dh)) v per query head, GQA (query head j reads kv head j / (Hq / Hkv)),
 // causal, optional sliding window -- the attention of the decoder-only models of Section 3.
 //
-// Decode (k_decode_attn): one CTA per (kv head, slot, KV split of 512 positions); the CTA serves
+// Decode, default for 16-bit KV with head_dim 128 and 8 kv heads: k_prefix_attn reads the prompt pages every
+// candidate shares once per 128 query rows (mma.sync, partial slot 0), then k_decode_stream -- one persistent
+// CTA per SM, each streaming an equal share of all (row, page) work through a TMA-fed ring of whole pages,
+// one mma.sync consumer warp per kv head, rows cut by a share boundary merged in CTA order by their last
+// finisher (no inter-CTA wait) -- folds the prefix partial into each row's result.
+//
+// Decode, other shapes and SR_ATTN_STREAM=0 (k_decode_attn_tc for 16-bit KV with mma.sync, k_decode_attn for
+// fp32 KV): one CTA per (kv head, slot, KV split of 512 positions); the CTA serves
 // the G query heads of its kv head, so each K/V byte is read once per group.  A token's K (and V)
 // row of dh elements is read by dh*size/16 threads with one 16-byte load each (fully coalesced
 // within the 4 KB (bf16, dh 128) page block of that head); token groups stride over the split;
@@ -12,8 +19,10 @@
 // result does not depend on the batch it is in; a combine kernel merges split partials.
 //
 // Prefill (k_prefill_attn): flash-attention style over packed variable-length sequences with a
-// shared prefix (the prompt's KV) -- 64 query rows x one head per CTA, 64-key blocks staged by
-// cp.async, bf16 mma.sync m16n8k16 with fp32 accumulation, online softmax in registers.
+// shared prefix (the prompt's KV) and, for the reward model with its cache, cached keys read from pages --
+// 64 query rows x one head per CTA, 64-key blocks staged by cp.async, 16-bit mma.sync m16n8k16 with fp32
+// accumulation, online softmax in registers.  Opt-in tcgen05 forms of the prefix pass and the prefill
+// (SR_PREFIX_TC=1, SR_PREFILL_TC=1) keep S and O in TMEM; they are parity-tested and measured slower.
 #include <algorithm>
 #include <mutex>
 #include <type_traits>
