@@ -1,10 +1,11 @@
 // libsr runtime: model loading, workspace, the generator / reward-model forward passes, and the
 // Speculative Rejection controller (Algorithm 1, Section 4.2) behind the C ABI of sr.h.
 //
-// Host code here only enqueues kernels and reads a handful of control words per step (live
-// count, free pages) to size the next launch; every step of the method runs on the device:
-// embedding, norms, GEMMs, RoPE + paged KV append, attention, sampling, partial-reward scoring,
-// the r_cut radix select, compaction and page release.
+// Host code here only enqueues kernels and reads a handful of control words (live count, free pages) to size
+// launches; between page boundaries, where no memory trigger can fire, decode steps are enqueued back to back
+// and the words are read once per boundary.  Every step of the method runs on the device: embedding, norms,
+// GEMMs, RoPE + paged KV append, attention, sampling, partial-reward scoring (with the reward model's K/V kept
+// across rounds when sr_set_rm_cache gives it a pool), the r_cut radix select, compaction and page release.
 #include <algorithm>
 #include <chrono>
 #include <cmath>
