@@ -49,6 +49,21 @@ def load_peaks():
         return {}
 
 
+def aggregate_over_ranks(maxes, sums, world, device="cpu"):
+    """Whole-job figures of one replica per rank: the max over ranks of each value in `maxes` (timed regions) and
+    the sum over ranks of each value in `sums` (work done).  world <= 1 returns them unchanged."""
+    maxes, sums = [float(x) for x in maxes], [float(x) for x in sums]
+    if world <= 1:
+        return maxes, sums
+    import torch
+    import torch.distributed as dist
+    tm = torch.tensor(maxes, dtype=torch.float64, device=device)
+    ts = torch.tensor(sums, dtype=torch.float64, device=device)
+    dist.all_reduce(tm, op=dist.ReduceOp.MAX)
+    dist.all_reduce(ts, op=dist.ReduceOp.SUM)
+    return [float(x) for x in tm.tolist()], [float(x) for x in ts.tolist()]
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -361,13 +376,8 @@ def main():
     ms = ev0.elapsed_time(ev1)
     gen_tokens = sum(s["gen_tokens"] for s in stats)
     rm_tokens = sum(s["rm_tokens"] for s in stats)
-    t = torch.tensor([ms, gen_tokens, rm_tokens], dtype=torch.float64, device="cuda")
-    if world > 1:
-        tmax = t.clone()
-        dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
-        tsum = t.clone()
-        dist.all_reduce(tsum, op=dist.ReduceOp.SUM)
-        ms, gen_tokens, rm_tokens = float(tmax[0]), float(tsum[1]), float(tsum[2])
+    (ms,), (gen_tokens, rm_tokens) = aggregate_over_ranks([ms], [gen_tokens, rm_tokens], world,
+                                                         "cuda" if world > 1 else "cpu")
     value = gen_tokens / (ms / 1e3)
 
     # end to end through the public host API: prompt H2D and result D2H inside the timed region
@@ -376,6 +386,8 @@ def main():
         sr.sr_set_profiling(ctx, False)
         hp = [w.prompt(i) for i in range(n_prompts)]
         torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
         t0 = time.perf_counter()
         e2e_tokens, h2d, d2h = 0, 0, 0
         for k in range(args.e2e_steps):
@@ -386,6 +398,9 @@ def main():
             h2d += p.nbytes
             d2h += toks.nbytes + 8
         dt = time.perf_counter() - t0
+        if world > 1:  # whole job: the slowest rank's wall time, every rank's tokens
+            dist.barrier()
+            (dt,), (e2e_tokens,) = aggregate_over_ranks([dt], [e2e_tokens], world, "cuda")
         e2e = {"value": e2e_tokens / dt, "unit": UNIT, "h2d_bytes_per_step": h2d // args.e2e_steps,
                "d2h_bytes_per_step": d2h // args.e2e_steps, "steps": args.e2e_steps,
                "ms_per_step": dt * 1e3 / args.e2e_steps}
