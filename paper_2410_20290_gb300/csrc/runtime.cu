@@ -16,11 +16,22 @@
 #include <cstdlib>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 
 namespace sr {
 
 static thread_local std::string g_msg;
+
+// NVTX range on the host timeline around one phase of the controller (prompt prefill, a decode step, a scoring
+// pass, a rejection round, the final scoring); a no-op unless a profiler such as Nsight Systems is attached.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 sr_status set_err(sr_status s, const char* fmt, ...) {
   char buf[1024];
@@ -682,6 +693,7 @@ sr_status upload_single_plan(sr_ctx* c, int P, PrefillPlan& plan) {
 // Prompt through the reward model (KV kept for every later scoring chunk) and through the
 // generator (KV into the shared pages + tail template page; logits of the last position).
 sr_status prefill_prompt(sr_ctx* c, sr_batch& b) {
+  NvtxRange nv("sr prefill");
   const Model& g = c->gen;
   const Model& r = c->rm;
   const int P = b.P;
@@ -765,6 +777,7 @@ sr_status admit(sr_ctx* c, sr_batch& b, int start, int count) {
 // b.n_live, an upper bound of the live count (candidates only complete between rounds), and the kernels
 // that write candidate state skip the slots past the device's live count.
 sr_status decode_step(sr_ctx* c, sr_batch& b, float* logits_host, bool sync = true) {
+  NvtxRange nv("sr decode step");
   const Model& m = c->gen;
   const sr_model_desc& d = m.d;
   Work& w = c->wg;
@@ -911,6 +924,7 @@ void rm_cache_release(RmCache& rc, const std::vector<char>& keep) {
 // can serve, in ascending id order, so that a later round or the final scoring reads them.
 sr_status score(sr_ctx* c, sr_batch& b, const std::vector<int>& ids_h, const std::vector<int>& taus,
                 float* rewards_dev, bool store, long long* rm_rows = nullptr) {
+  NvtxRange nv("sr score");
   const Model& r = c->rm;
   const int n = (int)ids_h.size();
   if (n == 0) return SR_OK;
@@ -1154,6 +1168,7 @@ sr_status begin(sr_ctx* c, sr_batch& b, const int32_t* prompt, bool prompt_on_de
 
 // Algorithm 1 for a prepared batch; outputs stay on the device (c->out_tok, d_outlen, d_score).
 sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, sr_stats* st) {
+  NvtxRange nv("sr generate");
   const bool pool_mode = sched->kind == SR_SCHED_POOL_FULL;
   std::vector<int> taus_sched(sched->tau, sched->tau + (sched->kind == SR_SCHED_FIXED ? sched->n_tau : 0));
   sr_stats S;
@@ -1197,6 +1212,7 @@ sr_status run_sr(sr_ctx* c, sr_batch& b, float alpha, const sr_schedule* sched, 
           double tsel = now_ms();
           S.ms_score += tsel - ts;
           {
+            NvtxRange nv("sr reject and compact");
             Scope sc(&c->prof, SR_KC_CONTROL, c->st);
             SR_TRY(ctl_round(b.P, b.n_sh, alpha, pool_mode && need ? 1 : 0, c->rr, c->rset, c->live, c->ctrl,
                              c->ctrlf, c->status, c->len, c->reward, c->pt, b.max_pages, c->free_stack, nullptr,
